@@ -72,7 +72,12 @@ def fit_latency(ns, attn_times, mlp_times):
 
 
 def round_half_away(x: float) -> int:
-    return int(np.floor(x + 0.5)) if x >= 0 else -int(np.floor(-x + 0.5))
+    """Nearest integer, halves away from zero (exact for every double: the
+    fractional part x - floor(x) is computed without rounding)."""
+    a = abs(float(x))
+    f = np.floor(a)
+    r = int(f) + (1 if a - f >= 0.5 else 0)
+    return r if x >= 0 else -r
 
 
 def integer_weights(ta: float, tm: float) -> tuple:
@@ -109,15 +114,18 @@ def knapsack(weights, values, budget: int):
     N = len(w)
     if budget < 0:
         raise ValueError("budget must be >= 0")
-    best = [0] * (budget + 1)
-    take = [[False] * (budget + 1) for _ in range(N)]
+    best = np.zeros(budget + 1, np.int64)
+    take = np.zeros((N, budget + 1), bool)
     for i in range(N):
-        new = list(best)
-        for c in range(w[i], budget + 1):
-            cand = best[c - w[i]] + q[i]
-            if cand > best[c]:
-                new[c] = cand
-                take[i][c] = True
+        # every capacity c >= w_i at once (Sec. 3.4: independent across the budget axis)
+        wi = w[i]
+        if wi > budget:
+            continue
+        cand = best[: budget + 1 - wi] + q[i]
+        upd = cand > best[wi:]
+        new = best.copy()
+        new[wi:][upd] = cand[upd]
+        take[i, wi:] = upd
         best = new
     mask = np.zeros(N, np.uint8)
     c = budget
@@ -125,7 +133,7 @@ def knapsack(weights, values, budget: int):
         if take[i][c]:
             mask[i] = 1
             c -= w[i]
-    return mask, best[budget]
+    return mask, int(best[budget])
 
 
 def knapsack_brute(weights, values, budget: int):

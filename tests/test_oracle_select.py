@@ -88,6 +88,9 @@ def test_integer_weights_table3_golden():
 
 def test_round_half_away():
     assert [S.round_half_away(v) for v in (0.5, 1.5, 2.5, -0.5, -1.5, 2.4999)] == [1, 2, 3, -1, -2, 2]
+    # the largest double below 0.5 rounds to 0 (x + 0.5 would round up to 1.0)
+    assert S.round_half_away(np.nextafter(0.5, 0.0)) == 0
+    assert S.round_half_away(2.0 ** 52 + 1) == 2 ** 52 + 1
 
 
 def test_sublayer_units_alternate_attn_mlp():
