@@ -1,0 +1,337 @@
+#!/usr/bin/env python3
+"""Accepted tokens/s of KnapSpec self-speculative decoding on one GB300.
+
+A step is one pass of the whole hot path on one sequence: gamma skip-masked
+draft steps (a1), the gamma+1-row verify pass with greedy acceptance (a2, a3),
+the history cosines (a4) and the knapsack mask selection (a5, re-solved every
+step).  `value` = accepted tokens (a + 1 per step) / device time of K steps;
+`e2e` = the same through ks_generate_speculative with host output buffers,
+wall clock.  Weights and prompts are seeded synthetic inputs (random-init
+model shapes, uniform random token ids).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload llama8b-4k]
+  python bench.py --impl reference ...   # the CPU oracle, same metric
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from paper_2602_20217_gb300.configs import WORKLOADS  # noqa: E402
+
+METRIC = "accepted tokens/sec at batch 1 on 1xGB300; decode-step HBM GB/s vs ~8 TB/s peak"
+UNIT = "tokens/s"
+DEFAULT_WORKLOAD = "llama8b-4k"
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+# ------------------------------------------------------------ oracle arm
+def oracle_sample_seconds(workload: str, seed: int = 0) -> dict:
+    """Time the fp64 oracle on a bounded sample of one greedy decode token:
+    layer 0's Attn + MLP sublayers at the workload's context (synthetic KV
+    cache) and 1/32 of the LM head rows; the token time is scaled to all
+    layers and the full vocabulary."""
+    from oracle import decoder as D
+    from paper_2602_20217_gb300 import synth
+    wl = WORKLOADS[workload]
+    sh = wl.shape
+    cfg = D.OracleConfig.like(sh)
+    lw = {k: synth.np_weight(sh, seed, 0, k).astype(np.float64) for k in synth.weight_shapes(sh)["layer"]}
+    n = wl.prompt_len
+    rng_key = synth.stream_key(seed, 0, "kv")
+    kv = synth.np_normal32(rng_key, np.arange(2 * sh.n_kv_heads * (n + 1) * sh.head_dim, dtype=np.uint64), 1.0)
+    kv = kv.astype(np.float64).reshape(2, sh.n_kv_heads, n + 1, sh.head_dim)
+    K, V = kv[0].copy(), kv[1].copy()
+    x = synth.np_weight_rows(sh, seed, 0, "embed", [7]).astype(np.float64)
+    rows = np.arange(0, sh.vocab, 32)
+    W_lm = synth.np_weight_rows(sh, seed, 0, "lm_head", rows).astype(np.float64)
+    gain = np.ones(sh.d_model)
+    t0 = time.perf_counter()
+    x1 = D.attn_sublayer(cfg, lw, x, np.array([n]), K, V)
+    x2 = D.mlp_sublayer(cfg, lw, x1)
+    t1 = time.perf_counter()
+    _ = D.rms_norm(x2, gain, cfg.rms_eps) @ W_lm.T
+    t2 = time.perf_counter()
+    return {"t_layer": t1 - t0, "t_lm_slice": t2 - t1,
+            "t_token": sh.n_layers * (t1 - t0) + (sh.vocab / len(rows)) * (t2 - t1)}
+
+
+def run_oracle_arm(args, workload):
+    """Runs in a child process with a fixed BLAS thread count; prints JSON."""
+    samples = []
+    for i in range(args.warmup + args.steps):
+        r = oracle_sample_seconds(workload)
+        if i >= args.warmup:
+            samples.append(r["t_token"])
+    return float(np.mean(samples))
+
+
+def cpu_baseline(workload: str, steps: int = 1, warmup: int = 0) -> dict:
+    cores = os.cpu_count() or 1
+    env = dict(os.environ)
+    for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        env[k] = str(cores)
+    code = ("import sys, json; sys.path.insert(0, %r); import bench; "
+            "print(json.dumps(bench.run_oracle_arm(type('A', (), {'steps': %d, 'warmup': %d})(), %r)))"
+            % (ROOT, steps, warmup, workload))
+    out = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True, timeout=900)
+    if out.returncode != 0:
+        raise RuntimeError("oracle baseline failed: " + out.stderr[-2000:])
+    t_token = float(out.stdout.strip().splitlines()[-1])
+    sh = WORKLOADS[workload].shape
+    return {"value": 1.0 / t_token, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": (f"fp64 numpy oracle, greedy decode token at {WORKLOADS[workload].prompt_len} context: "
+                       f"layer 0 Attn+MLP (synthetic KV) x {sh.n_layers} layers + 1/32 of LM-head rows x 32; "
+                       f"{steps} timed repeats; every emitted token counts as accepted")}
+
+
+def reference_arm(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    wl = args.workload
+    cb = cpu_baseline(wl, steps=args.steps, warmup=args.warmup)
+    line = {"metric": METRIC, "value": cb["value"], "unit": UNIT, "n_gpus": args.gpus, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": 1e3 / cb["value"], "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "impl": "reference",
+            "config": {"workload": wl, "model": WORKLOADS[wl].shape.name, "prompt": WORKLOADS[wl].prompt_len},
+            "cpu_baseline": cb,
+            "e2e": {"value": cb["value"], "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# --------------------------------------------------------------- GPU arm
+class ClockSampler:
+    def __init__(self, path):
+        self.path = path
+        self.proc = None
+
+    def __enter__(self):
+        q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={q}", "--format=csv,noheader,nounits",
+                                          "-lms", "200"], stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(5)
+            except Exception:
+                self.proc.kill()
+            self.f.close()
+
+    def summary(self, gpu_index: int):
+        try:
+            rows = [l.split(",") for l in open(self.path).read().strip().splitlines()]
+        except Exception:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        rows = [[c.strip() for c in r] for r in rows if r and r[0].strip() == str(gpu_index)]
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if len(r) > 5 + i and r[5 + i] == "Active"})
+        return {"sm_mhz": float(np.median(sm)) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+def gpu_arm(args):
+    import torch
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    from paper_2602_20217_gb300 import build, knapspec as ks, synth
+    from paper_2602_20217_gb300.model import Model
+    build.build()
+
+    wl = WORKLOADS[args.workload]
+    sh = wl.shape
+    gamma = args.gamma or wl.gammas[len(wl.gammas) // 2]
+    prompt = synth.prompt_tokens(sh, wl.prompt_len, seed=wl.prompt_seed)
+    max_seq = wl.prompt_len + (max(args.steps, args.warmup) + 2) * (gamma + 1) + args.e2e_tokens + 64
+    t0 = time.time()
+    model = Model(sh, max_seq=max_seq, seed=wl.weight_seed)
+    torch.cuda.synchronize()
+    t_setup = time.time() - t0
+    stream, h = model.stream, model.h
+
+    def prefill():
+        t = time.time()
+        model.prefill(prompt)
+        torch.cuda.synchronize()
+        return time.time() - t
+
+    # Latency model of App. C measured on this GPU at the prompt's context:
+    # c1 = MLP sublayer (gate/up + down), c3 = the Attn sublayer's
+    # context-independent kernels (QKV, merge, O-proj), c2 = attention-kernel
+    # time / context length.
+    t_prefill = prefill()
+    for k in range(9):
+        ks.ks_kernel_timing(h, k, True)
+    model.decode_greedy(8)
+    kt = {name: ks.ks_kernel_time(h, k) for name, k in ks.KLASS.items()}
+    for k in range(9):
+        ks.ks_kernel_timing(h, k, False)
+    per = lambda name: kt[name][1] / max(1, kt[name][0])
+    c1 = per("gateup") + per("down")
+    c3 = per("qkv") + per("merge") + per("oproj")
+    c2 = per("attn") / wl.prompt_len
+    lat, _keep = ks.latency(0, c1, c2, c3)
+
+    def params(max_steps):
+        return ks.KsSpecParams(gamma, 1, None, lat, float(args.budget_frac), int(args.resolve_every),
+                               int(max_steps))
+
+    # warm-up
+    prefill()
+    ks.ks_generate_speculative(h, params(args.warmup), 1 << 30)
+    # timed region: exactly K speculation steps, device time on the model's stream
+    prefill()
+    ks.ks_kernel_timing(h, ks.KLASS["gateup"], True)
+    launches0 = ks.ks_launch_count(h)
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    ev0 = torch.cuda.Event(enable_timing=True)
+    ev1 = torch.cuda.Event(enable_timing=True)
+    clk_path = (os.path.join(ROOT, "gpurun_out", f"clocks_rank{rank}.csv")
+                if os.path.isdir(os.path.join(ROOT, "gpurun_out")) else f"/tmp/ks_clocks_{rank}.csv")
+    clocks = ClockSampler(clk_path)
+    with clocks:
+        ev0.record(stream)
+        _, st, acc = ks.ks_generate_speculative(h, params(args.steps), 1 << 30)
+        ev1.record(stream)
+        torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    ms = ev0.elapsed_time(ev1)
+    launches = ks.ks_launch_count(h) - launches0
+    gu_n, gu_ms = ks.ks_kernel_time(h, ks.KLASS["gateup"])
+    ks.ks_kernel_timing(h, ks.KLASS["gateup"], False)
+    tokens = int(st.steps + st.accepted)
+
+    # e2e: the public call with host output buffers, wall clock, for a
+    # generation job of e2e_tokens tokens (the prompt already prefilled)
+    prefill()
+    h2d0, d2h0 = ks.ks_transfer_bytes(h)
+    t0 = time.perf_counter()
+    out, est, eacc = ks.ks_generate_speculative(h, params(0), args.e2e_tokens)
+    e2e_s = time.perf_counter() - t0
+    h2d1, d2h1 = ks.ks_transfer_bytes(h)
+    e2e_tok = int(est.steps + est.accepted)
+    # the same library's plain greedy decode of the same job
+    prefill()
+    t0 = time.perf_counter()
+    ar = ks.ks_decode_greedy(h, args.e2e_tokens)
+    ar_s = time.perf_counter() - t0
+    lossless = bool(np.array_equal(out, ar))
+
+    vals = torch.tensor([ms, float(tokens)], dtype=torch.float64, device="cuda")
+    if dist:
+        a = vals[0:1].clone()
+        b = vals[1:2].clone()
+        dist.all_reduce(a, op=dist.ReduceOp.MAX)
+        dist.all_reduce(b, op=dist.ReduceOp.SUM)
+        vals = torch.cat([a, b])
+    ms_max, tok_all = float(vals[0]), float(vals[1])
+
+    if rank == 0:
+        peak, peak_kind = peaks()
+        gu_bytes = 2 * sh.d_ff * sh.d_model * sh.elem_bytes   # weight bytes one gate/up launch must read
+        gu_avg_ms = gu_ms / max(1, gu_n)
+        achieved = gu_bytes / (gu_avg_ms * 1e-3) / 1e9
+        line = {
+            "metric": METRIC, "value": tok_all / (ms_max * 1e-3), "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_max / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": sh.dtype,
+            "data": "synthetic (seeded random-init weights, uniform random prompt ids)",
+            "config": {"workload": wl.name, "model": sh.name, "prompt": wl.prompt_len, "gamma": gamma,
+                       "policy": (f"knapsack re-solved every {args.resolve_every} step(s), "
+                                  f"budget {args.budget_frac} of sum w"),
+                       "l2": "inputs larger than L2 (each step streams the weights, 16+ GB)",
+                       "parallelism": f"replicas x{world}"},
+            "tokens": tokens, "mean_tokens_per_step": tokens / max(1, st.steps),
+            "alpha": float(st.accepted) / max(1, st.drafted),
+            "mask_skipped": {"attn": int(st.attn_skipped), "mlp": int(st.mlp_skipped)},
+            "ar_tokens_per_s": (args.e2e_tokens - 1) / ar_s,
+            "spec_vs_ar_e2e": (e2e_tok / e2e_s) / ((args.e2e_tokens - 1) / ar_s),
+            "lossless_vs_ar": lossless,
+            "latency_model_ms": {"c1": c1, "c2": c2, "c3": c3},
+            "prefill_s": t_prefill, "setup_s": t_setup,
+            "e2e": {"value": e2e_tok / e2e_s, "unit": UNIT,
+                    "h2d_bytes_per_step": (h2d1 - h2d0) / max(1, est.steps),
+                    "d2h_bytes_per_step": (d2h1 - d2h0) / max(1, est.steps)},
+            "gpu_launches": launches,
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                         "frac": achieved / peak, "traffic": None,
+                         "kernel": "gemv_kernel SwiGLU (gate/up)", "peak_source": peak_kind,
+                         "launches_timed": gu_n, "bytes_per_launch": gu_bytes},
+            "kernels_us": {k: round(1e3 * v[1] / max(1, v[0]), 2) for k, v in kt.items()},
+            "clocks": clocks.summary(local),
+        }
+        if not args.no_cpu_baseline and world == 1:
+            try:
+                line["cpu_baseline"] = cpu_baseline(wl.name)
+            except Exception as e:  # reported, never hidden
+                line["cpu_baseline"] = {"error": str(e)[:300]}
+        print(json.dumps(line), flush=True)
+    model.close()
+    if dist:
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=48)
+    ap.add_argument("--warmup", type=int, default=4)
+    ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(WORKLOADS))
+    ap.add_argument("--gamma", type=int, default=0)
+    ap.add_argument("--budget-frac", dest="budget_frac", type=float, default=0.8)
+    ap.add_argument("--resolve-every", dest="resolve_every", type=int, default=1)
+    ap.add_argument("--e2e-tokens", dest="e2e_tokens", type=int, default=256)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    if args.impl == "reference":
+        reference_arm(args)
+    else:
+        gpu_arm(args)
+
+
+if __name__ == "__main__":
+    main()

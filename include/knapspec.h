@@ -1,0 +1,271 @@
+/*
+ * knapspec.h - C ABI of a single-GPU (GB300, sm_103a) implementation of the
+ * data-parallel hot path of KnapSpec self-speculative decoding
+ * (Cha, Kim, Han, Yang, Han: "KnapSpec: Self-Speculative Decoding via
+ * Adaptive Layer Selection as a Knapsack Problem", arXiv 2602.20217).
+ *
+ * The hot path, per speculation step:
+ *   a1  draft:   gamma greedy tokens from the skip-masked sub-network f^(S)
+ *                (Sec. 2: f^(S) composes the sublayers in S in their order;
+ *                f^(2i-1) = Attn_i, f^(2i) = MLP_i, norms included);
+ *   a2  verify:  the full target f over the gamma+1 rows in one pass (Sec. 2.1);
+ *   a3  accept:  greedy acceptance - keep drafts while they equal the target's
+ *                argmax, then append the target's own token (Sec. 2.1, Eq. 1);
+ *   a4  cosine:  per-sublayer matrix cosines of the history hidden states
+ *                (Sec. 2 definition of cos(X, Y); Sec. 3.4, m = 5 steps);
+ *   a5  select:  integer latency weights (Sec. 3.4, App. C) and an exact 0/1
+ *                knapsack over the 2L sublayers (Sec. 3.3) -> next draft mask.
+ *
+ * Conventions for every call:
+ *  - All device memory is allocated by the caller.  The library borrows
+ *    pointers and never frees them.  A model handle owns host metadata, a
+ *    small pinned host staging buffer and CUDA events only.
+ *  - "dev" pointers are device addresses; "host" pointers are host memory.
+ *  - Weights are row-major [out, in] (y = W x), dtype KS_DTYPE_F32 or
+ *    KS_DTYPE_BF16; norm gains have the same dtype.  The residual stream and
+ *    all reductions are fp32; bf16 models feed bf16 activations to the
+ *    matrix products and keep the KV cache in bf16.
+ *  - Every call returns a ks_status and never aborts, traps or exits.
+ *    Invalid arguments are rejected before any work is enqueued.  CUDA errors
+ *    are reported as KS_ERR_CUDA (the message is kept per thread, see
+ *    ks_last_error).  No kernel spins on a flag; no call waits without a
+ *    bound other than a stream synchronisation.
+ *  - One handle is used by one host thread at a time and issues all work on
+ *    the stream given at creation.
+ *  - Greedy argmax ties resolve to the lowest token id.
+ */
+#ifndef KNAPSPEC_H
+#define KNAPSPEC_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    KS_OK = 0,
+    KS_ERR_INVALID_ARG = 1,   /* null/misaligned pointer, bad size, bad shape      */
+    KS_ERR_CUDA = 2,          /* a CUDA runtime call or kernel launch failed        */
+    KS_ERR_WORKSPACE = 3,     /* the workspace is smaller than required             */
+    KS_ERR_CAPACITY = 4,      /* KV capacity (max_seq) or row capacity exceeded     */
+    KS_ERR_TIMEOUT = 5,       /* reserved: a bounded device wait gave up            */
+    KS_ERR_UNSUPPORTED = 6,   /* shape/dtype outside what the kernels implement     */
+    KS_ERR_STATE = 7          /* call out of order (e.g. draft before prefill)      */
+} ks_status;
+
+enum { KS_DTYPE_F32 = 0, KS_DTYPE_BF16 = 1 };
+
+/* Decoder shape (Sec. 2 with the Llama / Qwen3 block; see the design notes).
+ * Supported: head_dim in {64, 128}; n_q_heads % n_kv_heads == 0;
+ * d_model, d_ff, head_dim multiples of 8; max_rows <= 16. */
+typedef struct {
+    int32_t n_layers;        /* L; the model has 2L sublayers                          */
+    int32_t d_model;
+    int32_t n_q_heads;
+    int32_t n_kv_heads;
+    int32_t head_dim;
+    int32_t d_ff;
+    int32_t vocab;
+    int32_t qk_norm;         /* 1: per-head RMSNorm on q and k before RoPE (Qwen3)     */
+    int32_t dtype;           /* KS_DTYPE_F32 or KS_DTYPE_BF16                          */
+    int32_t max_seq;         /* KV capacity in positions                               */
+    int32_t max_rows;        /* rows per pass: >= gamma + 1 and the prefill chunk      */
+    int32_t hist_steps;      /* m: speculation steps kept in the history (Sec. 3.4)    */
+    int32_t hist_init_rows;  /* prompt rows that seed the history at prefill           */
+    float rms_eps;
+    double rope_theta;       /* rotate-half RoPE, inv_freq_j = theta^(-2j/head_dim)    */
+} ks_config;
+
+/* Borrowed device pointers.  Per-layer fields point to host arrays of
+ * n_layers device pointers.  q_norm / k_norm may be NULL when qk_norm == 0.
+ *   embed      [vocab, d]           lm_head  [vocab, d]     final_norm [d]
+ *   attn_norm  [d]                  w_qkv    [(hq + 2 hk) hd, d]  (q; k; v rows)
+ *   w_o        [d, hq hd]           q_norm, k_norm [hd]
+ *   mlp_norm   [d]                  w_gate_up [2 d_ff, d]  (gate rows, then up rows)
+ *   w_down     [d, d_ff]
+ * Every device pointer must be 16-byte aligned. */
+typedef struct {
+    const void* embed;
+    const void* lm_head;
+    const void* final_norm;
+    const void* const* attn_norm;
+    const void* const* w_qkv;
+    const void* const* w_o;
+    const void* const* q_norm;
+    const void* const* k_norm;
+    const void* const* mlp_norm;
+    const void* const* w_gate_up;
+    const void* const* w_down;
+} ks_weights;
+
+/* Latency model used for the knapsack weights.
+ * kind 0: App. C model t_MLP = c1, t_Attn(n) = c2 n + c3, turned into integer
+ *         weights by Sec. 3.4: Delta = min(t_Attn(n), t_MLP),
+ *         w = round(t / Delta) (half away from zero, at least 1).
+ * kind 1: explicit integer units per sublayer, units[2L] (host), all >= 1. */
+typedef struct {
+    int32_t kind;
+    double c1, c2, c3;
+    const int32_t* units;
+} ks_latency;
+
+typedef struct ks_model ks_model;
+
+/* ------------------------------------------------------------ model (a1-a3) */
+
+/* Bytes of device workspace a model with this config needs (KV cache, RoPE
+ * table, activations, split partials, history ring).  0 on an invalid config. */
+size_t ks_workspace_bytes(const ks_config* cfg);
+
+/* Validate cfg, borrow the weights and the workspace (dev, 256-byte aligned,
+ * at least ks_workspace_bytes(cfg) bytes), build the RoPE table, and return a
+ * handle bound to `stream` (a cudaStream_t; NULL = legacy default stream).
+ * No decoding state exists until ks_prefill. */
+ks_status ks_model_create(const ks_config* cfg, const ks_weights* w, void* workspace,
+                          size_t workspace_bytes, void* stream, ks_model** out);
+ks_status ks_model_destroy(ks_model* m);
+
+/* Run the prompt (host int32[n], 1 <= n, n + 1 <= max_seq) through the target
+ * in chunks of max_rows rows, fill the KV cache, seed the history with the
+ * last hist_init_rows prompt rows, and set the pending token to the greedy
+ * next token, written to *next_token (host).  Resets any previous sequence. */
+ks_status ks_prefill(ks_model* m, const int32_t* tokens, int32_t n, int32_t* next_token);
+
+/* a1 (Sec. 2, Sec. 2.2): gamma (1 <= gamma < max_rows) greedy draft tokens
+ * from f^(S), S = { i : mask[i-1] != 0 } (host uint8[2L]; odd 1-based
+ * sublayers are Attn, even are MLP), starting from the pending token at the
+ * committed length p.  A skipped sublayer is the identity on the residual
+ * stream.  Run Attn sublayers write K/V at positions p.. (overwritten by the
+ * verify).  The drafts stay on the device; if draft_tokens (host int32[gamma])
+ * is not NULL the call also waits for them and copies them out. */
+ks_status ks_draft(ks_model* m, const uint8_t* mask, int32_t gamma, int32_t* draft_tokens);
+
+/* a2 + a3 (Sec. 2.1): score [pending, drafts...] (gamma + 1 rows at positions
+ * p..p+gamma) with the full target in one pass, take the greedy argmax of
+ * each row, accept the longest prefix of drafts equal to the target's
+ * argmaxes (a of them) and append the target's own next token.  Commits the
+ * a + 1 rows (p += a + 1), records their per-sublayer hidden states in the
+ * history ring, and makes the appended token pending.
+ * draft_tokens: host int32[gamma] to score, or NULL to score the drafts of the
+ * preceding ks_draft call with the same gamma.
+ * Outputs (host): *n_accepted = a; out_tokens[0..a] = the a + 1 new tokens
+ * (room for gamma + 1); *n_out = a + 1.  Waits for the stream. */
+ks_status ks_verify(ks_model* m, const int32_t* draft_tokens, int32_t gamma,
+                    int32_t* n_accepted, int32_t* out_tokens, int32_t* n_out);
+
+/* Plain greedy autoregressive decoding of n_tokens tokens with the full
+ * target (the non-speculative baseline).  out (host int32[n_tokens]) receives
+ * the pending token followed by the next n_tokens - 1 greedy tokens; the
+ * last one is left pending.  One host synchronisation at the end. */
+ks_status ks_decode_greedy(ks_model* m, int32_t n_tokens, int32_t* out);
+
+/* Committed length p and the pending token. */
+ks_status ks_model_position(const ks_model* m, int32_t* committed, int32_t* pending);
+
+/* ------------------------------------------------------------ cosine (a4) */
+
+/* Sec. 2 matrix cosine for n_pairs pairs of [rows, d] matrices:
+ *   out[p] = (1/rows) sum_i <X_p[i], Y_p[i]> / (|X_p[i]| |Y_p[i]|)
+ * X_p = X + p * pair_stride elements, Y_p likewise (row i at + i * d, or at
+ * + row_index[i] * d when row_index (dev int32[rows]) is not NULL).
+ * X, Y: dev, dtype KS_DTYPE_F32 or KS_DTYPE_BF16.  out: dev float[n_pairs].
+ * Each pair's row terms are summed in row order (deterministic).  A zero row
+ * gives a NaN term, as the definition does. */
+ks_status ks_cosine(const void* X, const void* Y, int32_t dtype, int64_t n_pairs,
+                    int32_t rows, int32_t d, int64_t pair_stride, const int32_t* row_index,
+                    float* out, void* stream);
+
+/* a4 for a model: sims (dev float[2L]) receive sigma_i = cos(X^(i-1), X^(i))
+ * over the rows held in the history ring (Sec. 3.4: the tokens of the last m
+ * speculation steps), i = 1..2L; *rows_used (host, optional) = r. */
+ks_status ks_history_similarities(ks_model* m, float* sims, int32_t* rows_used);
+
+/* ------------------------------------------------------------ select (a5) */
+
+/* Integer weights of the 2L sublayers at context length context_len
+ * (Sec. 3.4 / App. C, see ks_latency), then the exact 0/1 knapsack
+ *   maximise sum_{i in S} q_i  subject to  sum_{i in S} w_i <= budget_units,
+ * q_i = round((1 - sims[i-1]) * 2^30) as int64 (half away from zero, from the
+ * fp32 similarity in double): the similarity lost by skipping sublayer i.
+ * Among optimal masks the one with the smallest bitmask value (bit i-1 <->
+ * sublayer i) is returned, so the result is exact and reproducible.
+ * sims: dev float[n_sublayers].  Outputs (dev): mask_out uint8[n_sublayers]
+ * (1 = run), objective_out double (sum q_i / 2^30, may be NULL), weights_out
+ * int32[n_sublayers] (may be NULL).  n_sublayers even, 2..256;
+ * 0 <= budget_units <= 65535.  scratch (dev, 16-byte aligned) must hold
+ * ks_select_scratch_bytes(n_sublayers, budget_units) bytes; the call does not
+ * allocate. */
+size_t ks_select_scratch_bytes(int32_t n_sublayers, int32_t budget_units);
+ks_status ks_select_mask(const ks_latency* lat, const float* sims, int64_t context_len,
+                         int32_t n_sublayers, int32_t budget_units, uint8_t* mask_out,
+                         double* objective_out, int32_t* weights_out, void* scratch,
+                         size_t scratch_bytes, void* stream);
+
+/* ------------------------------------------------- full speculative loop */
+
+typedef struct {
+    int32_t gamma;           /* draft length per step (1 <= gamma < max_rows)              */
+    int32_t policy;          /* 0 fixed mask, 1 knapsack re-solved every resolve_every steps */
+    const uint8_t* mask;     /* host uint8[2L]: the mask for policy 0                      */
+    ks_latency latency;      /* policy 1                                                   */
+    double budget_frac;      /* policy 1: budget = floor(budget_frac * sum_i w_i)          */
+    int32_t resolve_every;   /* policy 1: optimisation interval T in verify steps (>= 1)   */
+    int32_t max_steps;       /* stop after this many verify steps (0: no limit)             */
+} ks_spec_params;
+
+typedef struct {
+    int64_t steps;           /* verify steps                                    */
+    int64_t drafted;         /* draft tokens proposed                           */
+    int64_t accepted;        /* draft tokens accepted                           */
+    int64_t resolves;        /* knapsack solves                                 */
+    int64_t attn_skipped;    /* sublayers skipped by the last mask: Attn / MLP  */
+    int64_t mlp_skipped;
+} ks_spec_stats;
+
+/* Greedy self-speculative decoding of n_tokens tokens: repeat a1..a5 until
+ * n_tokens tokens are known (the pending token counts as the first) or
+ * max_steps verify steps have run.  Tokens produced = 1 + steps + accepted.
+ * out: host int32[n_tokens].  The token stream equals ks_decode_greedy's.
+ * accepted_per_step (host int32[], optional, room for n_tokens entries). */
+ks_status ks_generate_speculative(ks_model* m, const ks_spec_params* params, int32_t n_tokens,
+                                  int32_t* out, ks_spec_stats* stats, int32_t* accepted_per_step);
+
+/* ------------------------------------------------------------ diagnostics */
+
+/* Copy a window of device state to the caller (for tests):
+ * what = 0: logits of the last pass, float[rows][vocab];
+ *        1: the residual stream rows, float[rows][d];
+ *        2: K cache of layer `layer`, [n_kv_heads][positions][head_dim] in the model dtype
+ *           for positions [start, start + count), dst laid out [hk][count][hd];
+ *        3: V cache, as 2;
+ *        4: history ring states of the committed rows, float[2L+1][r][d], with
+ *           count == r; count == 0 writes r itself (int32) to dst;
+ * dst is host memory of `bytes` bytes; the call waits for the stream. */
+ks_status ks_debug_read(ks_model* m, int32_t what, int32_t layer, int32_t start, int32_t count,
+                        void* dst, size_t bytes);
+
+/* Per-kernel timing with CUDA events on the model's stream.  While enabled,
+ * every launch of the kernel class `klass` (0 QKV, 1 attention, 2 merge,
+ * 3 O-proj, 4 gate/up, 5 down, 6 LM head, 7 embed, 8 accept) is bracketed
+ * by events; ks_kernel_time returns the launches and total milliseconds
+ * since enabling.  Enabling resets the counters. */
+ks_status ks_kernel_timing(ks_model* m, int32_t klass, int32_t enable);
+ks_status ks_kernel_time(ks_model* m, int32_t klass, int64_t* launches, double* total_ms);
+
+/* Launch counter: kernels this handle has launched since creation. */
+int64_t ks_launch_count(const ks_model* m);
+
+/* Bytes this handle has copied host->device and device->host since creation
+ * (prompt and draft uploads, history row lists, results, masks, tokens). */
+ks_status ks_transfer_bytes(const ks_model* m, int64_t* h2d, int64_t* d2h);
+
+const char* ks_status_str(ks_status s);
+/* Last error message of the calling thread ("" if none). */
+const char* ks_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* KNAPSPEC_H */

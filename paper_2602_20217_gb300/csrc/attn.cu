@@ -1,0 +1,449 @@
+// Causal GQA attention over the KV cache for R <= 16 query rows (the Attn
+// sublayer of Sec. 2 inside a draft step or the gamma+1-row verify pass).
+//
+// Split-KV ("flash-decode"): one CTA per (KV head, chunk of kAttnChunk keys).
+// Chunk boundaries are absolute key positions and each chunk is split into
+// four fixed 32-key warp ranges merged in warp order, so the arithmetic
+// applied to one query row does not depend on how many rows share the pass:
+// keys past a row's own position are masked to -inf (their exp2 is exactly 0)
+// and chunks past it are skipped by the merge.  Greedy decoding and the
+// verify pass therefore produce bit-identical attention outputs.
+//
+// Per CTA: the new rows' K (QK-RMSNorm, RoPE) and V are written to the cache
+// by the CTA whose chunk holds their position, the G x R query vectors are
+// normalised, rotated and pre-scaled by log2(e)/sqrt(hd); K/V of the chunk are
+// staged in shared memory with cp.async (zero-filled past the valid keys).
+// bf16 models: S = Q K^T and O += P V on mma.sync.m16n8k16 with fp32 online
+// softmax in the log2 domain.  fp32 models: CUDA-core dot products.
+// Partials (m, l, o) per (row, query head, chunk) are merged in chunk order
+// by attn_merge_kernel.
+#include "common.cuh"
+#include "internal.h"
+
+namespace ks {
+
+constexpr int kAttnWarps = 4;
+constexpr float kLog2e = 1.4426950408889634f;
+
+// ------------------------------------------------------------ small helpers
+KS_DEV void cp_async16(void* smem, const void* gmem, bool valid) {
+    const uint32_t s = (uint32_t)__cvta_generic_to_shared(smem);
+    const int n = valid ? 16 : 0;
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(s), "l"(gmem), "r"(n));
+}
+KS_DEV void cp_async_wait_all() { asm volatile("cp.async.wait_all;\n" ::); }
+
+KS_DEV void ldmatrix_x4(uint32_t (&r)[4], const void* p) {
+    const uint32_t s = (uint32_t)__cvta_generic_to_shared(p);
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];\n"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(s));
+}
+KS_DEV void ldmatrix_x4_trans(uint32_t (&r)[4], const void* p) {
+    const uint32_t s = (uint32_t)__cvta_generic_to_shared(p);
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];\n"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(s));
+}
+
+// Load one head vector (hd = 32 * NPL elements) of row r from the fp32
+// projections, apply optional RMSNorm with gain, then rotate-half RoPE at
+// position pos.  Lane l holds elements l + 32 i.
+template <typename WT, int NPL>
+KS_DEV void head_vector(const float* src, const WT* gain, float eps, const float* rope, int pos,
+                        float (&v)[NPL]) {
+    const int lane = threadIdx.x & 31;
+    constexpr int hd = 32 * NPL;
+#pragma unroll
+    for (int i = 0; i < NPL; ++i) v[i] = src[lane + 32 * i];
+    if (gain != nullptr) {
+        float ss = 0.f;
+#pragma unroll
+        for (int i = 0; i < NPL; ++i) ss = fmaf(v[i], v[i], ss);
+        ss = warp_sum(ss);
+        const float inv = rsqrtf(ss / (float)hd + eps);
+#pragma unroll
+        for (int i = 0; i < NPL; ++i) v[i] = (v[i] * inv) * to_float(gain[lane + 32 * i]);
+    }
+    const float* rp = rope + (size_t)pos * hd;  // [hd/2][2]
+#pragma unroll
+    for (int i = 0; i < NPL / 2; ++i) {
+        const int j = lane + 32 * i;
+        const float c = rp[2 * j], s = rp[2 * j + 1];
+        const float a = v[i], b = v[i + NPL / 2];
+        v[i] = a * c - b * s;
+        v[i + NPL / 2] = b * c + a * s;
+    }
+}
+
+// Prologue shared by both kernels: write this chunk's new K/V rows to the
+// cache and return the valid key range [cs, ce).
+template <typename WT, int NPL>
+KS_DEV void write_new_kv(const AttnArgs& a, int h, int cs, int ce) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    constexpr int hd = 32 * NPL;
+    WT* kc = reinterpret_cast<WT*>(a.kcache) + (size_t)h * a.max_seq * hd;
+    WT* vc = reinterpret_cast<WT*>(a.vcache) + (size_t)h * a.max_seq * hd;
+    const WT* kn = reinterpret_cast<const WT*>(a.k_norm);
+    for (int r = warp; r < a.R; r += kAttnWarps) {
+        const int pos = a.p0 + r;
+        if (pos < cs || pos >= ce) continue;
+        const float* row = a.qkv + (size_t)r * a.qkv_ld;
+        float k[NPL];
+        head_vector<WT, NPL>(row + (a.hq + h) * hd, kn, a.eps, a.rope, pos, k);
+        const float* vsrc = row + (a.hq + a.hk + h) * hd;
+#pragma unroll
+        for (int i = 0; i < NPL; ++i) {
+            kc[(size_t)pos * hd + lane + 32 * i] = from_float<WT>(k[i]);
+            vc[(size_t)pos * hd + lane + 32 * i] = from_float<WT>(vsrc[lane + 32 * i]);
+        }
+    }
+}
+
+// ----------------------------------------------------------- bf16 kernel
+// Shared layout (bf16, row pitch hd + 8 elements = 16 B padding):
+//   Qs [mpad][P]  Ks [C][P]  Vs [C][P]   then fp32 warp partials.
+template <int HD>
+__global__ void __launch_bounds__(128) attn_bf16_kernel(const AttnArgs a) {
+    constexpr int NPL = HD / 32;
+    constexpr int P = HD + 8;
+    constexpr int C = kAttnChunk;
+    constexpr int KW = C / kAttnWarps;  // keys per warp (32)
+    constexpr int NDT = HD / 8;         // dim tiles of 8
+    extern __shared__ __align__(16) unsigned char smem[];
+
+    const int h = blockIdx.x, c = blockIdx.y;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int g = lane >> 2, t = lane & 3;
+    const int G = a.hq / a.hk;
+    const int M = G * a.R;
+    const int mtiles = (M + 15) >> 4;
+    const int mpad = mtiles * 16;
+    const int cs = c * C;
+    const int ce = min(cs + C, a.p0 + a.R);
+
+    __nv_bfloat16* Qs = reinterpret_cast<__nv_bfloat16*>(smem);
+    __nv_bfloat16* Ks = Qs + (size_t)mpad * P;
+    __nv_bfloat16* Vs = Ks + (size_t)C * P;
+    float* wpart = reinterpret_cast<float*>(Vs + (size_t)C * P);  // [4][16][HD + 2]
+
+    // 1. new K/V rows of this chunk -> cache (generic stores, then barrier)
+    write_new_kv<__nv_bfloat16, NPL>(a, h, cs, ce);
+    __syncthreads();
+
+    // 2. stage K/V of keys [cs, ce) (zero past ce)
+    const __nv_bfloat16* kg = reinterpret_cast<const __nv_bfloat16*>(a.kcache) + ((size_t)h * a.max_seq + cs) * HD;
+    const __nv_bfloat16* vg = reinterpret_cast<const __nv_bfloat16*>(a.vcache) + ((size_t)h * a.max_seq + cs) * HD;
+    constexpr int CPR = HD / 8;  // 16-byte chunks per row
+    for (int i = tid; i < C * CPR; i += blockDim.x) {
+        const int row = i / CPR, col = (i - row * CPR) * 8;
+        const bool ok = cs + row < ce;
+        const size_t off = ok ? (size_t)row * HD + col : 0;
+        cp_async16(Ks + row * P + col, kg + off, ok);
+        cp_async16(Vs + row * P + col, vg + off, ok);
+    }
+
+    // 3. queries: m = r * G + gq, scaled into the log2 domain, bf16
+    const float qscale = kLog2e * rsqrtf((float)HD);
+    const __nv_bfloat16* qn = reinterpret_cast<const __nv_bfloat16*>(a.q_norm);
+    for (int m = warp; m < mpad; m += kAttnWarps) {
+        if (m < M) {
+            const int r = m / G, gq = m - r * G;
+            float q[NPL];
+            head_vector<__nv_bfloat16, NPL>(a.qkv + (size_t)r * a.qkv_ld + (h * G + gq) * HD, qn, a.eps,
+                                            a.rope, a.p0 + r, q);
+#pragma unroll
+            for (int i = 0; i < NPL; ++i) Qs[m * P + lane + 32 * i] = __float2bfloat16_rn(q[i] * qscale);
+        } else {
+#pragma unroll
+            for (int i = 0; i < NPL; ++i) Qs[m * P + lane + 32 * i] = __float2bfloat16_rn(0.f);
+        }
+    }
+    cp_async_wait_all();
+    __syncthreads();
+
+    const int kbase = warp * KW;  // warp's key range within the chunk
+    for (int mt = 0; mt < mtiles; ++mt) {
+        // Q fragments of this m-tile
+        uint32_t qf[HD / 16][4];
+#pragma unroll
+        for (int ks = 0; ks < HD / 16; ++ks) {
+            const int mi = lane >> 3;
+            const int row = mt * 16 + (mi & 1) * 8 + (lane & 7);
+            const int col = ks * 16 + (mi >> 1) * 8;
+            ldmatrix_x4(qf[ks], Qs + row * P + col);
+        }
+        // row positions of the two rows this thread holds
+        int rpos[2];
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+            const int m = mt * 16 + g + 8 * hh;
+            rpos[hh] = (m < M) ? a.p0 + m / G : -1;  // padding rows see no key
+        }
+        float o[NDT][4];
+#pragma unroll
+        for (int i = 0; i < NDT; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
+        float mrow[2] = {-INFINITY, -INFINITY};
+        float lrow[2] = {0.f, 0.f};
+
+        for (int kt = 0; kt < KW; kt += 16) {
+            const int key0 = kbase + kt;  // within chunk
+            // S = Q K^T for 16 keys (two n-tiles of 8)
+            float s[2][4];
+#pragma unroll
+            for (int j = 0; j < 2; ++j) s[j][0] = s[j][1] = s[j][2] = s[j][3] = 0.f;
+#pragma unroll
+            for (int ks = 0; ks < HD / 16; ++ks) {
+                uint32_t kb[4];
+                // matrices: (keys 0-7, d 0-7), (keys 0-7, d 8-15), (keys 8-15, d 0-7), (keys 8-15, d 8-15)
+                const int mi = lane >> 3;
+                const int krow = key0 + (mi >> 1) * 8 + (lane & 7);
+                const int kcol = ks * 16 + (mi & 1) * 8;
+                ldmatrix_x4(kb, Ks + krow * P + kcol);
+                mma_bf16(s[0], qf[ks][0], qf[ks][1], qf[ks][2], qf[ks][3], kb[0], kb[1]);
+                mma_bf16(s[1], qf[ks][0], qf[ks][1], qf[ks][2], qf[ks][3], kb[2], kb[3]);
+            }
+            // causal / validity mask and online softmax (log2 domain)
+#pragma unroll
+            for (int hh = 0; hh < 2; ++hh) {
+                float tmax = -INFINITY;
+#pragma unroll
+                for (int j = 0; j < 2; ++j)
+#pragma unroll
+                    for (int e = 0; e < 2; ++e) {
+                        const int key = cs + key0 + j * 8 + 2 * t + e;
+                        float& v = s[j][2 * hh + e];
+                        if (key > rpos[hh] || key >= ce) v = -INFINITY;
+                        tmax = fmaxf(tmax, v);
+                    }
+                tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 1));
+                tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 2));
+                const float mnew = fmaxf(mrow[hh], tmax);
+                float alpha, psum = 0.f;
+                if (mnew == -INFINITY) {
+                    alpha = 1.f;
+#pragma unroll
+                    for (int j = 0; j < 2; ++j) s[j][2 * hh] = s[j][2 * hh + 1] = 0.f;
+                } else {
+                    alpha = exp2f(mrow[hh] - mnew);
+#pragma unroll
+                    for (int j = 0; j < 2; ++j)
+#pragma unroll
+                        for (int e = 0; e < 2; ++e) {
+                            float& v = s[j][2 * hh + e];
+                            v = exp2f(v - mnew);
+                            psum += v;
+                        }
+                }
+                mrow[hh] = mnew;
+                lrow[hh] = lrow[hh] * alpha + psum;
+#pragma unroll
+                for (int i = 0; i < NDT; ++i) {
+                    o[i][2 * hh] *= alpha;
+                    o[i][2 * hh + 1] *= alpha;
+                }
+            }
+            // O += P V
+            const uint32_t pa0 = pack_bf16(s[0][0], s[0][1]);
+            const uint32_t pa1 = pack_bf16(s[0][2], s[0][3]);
+            const uint32_t pa2 = pack_bf16(s[1][0], s[1][1]);
+            const uint32_t pa3 = pack_bf16(s[1][2], s[1][3]);
+#pragma unroll
+            for (int dp = 0; dp < NDT / 2; ++dp) {
+                uint32_t vb[4];
+                // matrices: (keys 0-7, d), (keys 8-15, d), (keys 0-7, d+8), (keys 8-15, d+8)
+                const int mi = lane >> 3;
+                const int vrow = key0 + (mi & 1) * 8 + (lane & 7);
+                const int vcol = dp * 16 + (mi >> 1) * 8;
+                ldmatrix_x4_trans(vb, Vs + vrow * P + vcol);
+                mma_bf16(o[2 * dp], pa0, pa1, pa2, pa3, vb[0], vb[1]);
+                mma_bf16(o[2 * dp + 1], pa0, pa1, pa2, pa3, vb[2], vb[3]);
+            }
+        }
+        // full row sums of l across the quad
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+            lrow[hh] += __shfl_xor_sync(0xffffffffu, lrow[hh], 1);
+            lrow[hh] += __shfl_xor_sync(0xffffffffu, lrow[hh], 2);
+        }
+        // warp partials -> shared
+        float* wp = wpart + (size_t)warp * 16 * (HD + 2);
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+            const int rr = g + 8 * hh;
+            if (t == 0) {
+                wp[rr * (HD + 2) + 0] = mrow[hh];
+                wp[rr * (HD + 2) + 1] = lrow[hh];
+            }
+#pragma unroll
+            for (int i = 0; i < NDT; ++i) {
+                wp[rr * (HD + 2) + 2 + i * 8 + 2 * t] = o[i][2 * hh];
+                wp[rr * (HD + 2) + 2 + i * 8 + 2 * t + 1] = o[i][2 * hh + 1];
+            }
+        }
+        __syncthreads();
+        // merge the four warp ranges in warp order -> global chunk partial
+        for (int idx = tid; idx < 16 * (HD + 2); idx += blockDim.x) {
+            const int rr = idx / (HD + 2), col = idx - rr * (HD + 2);
+            const int m = mt * 16 + rr;
+            if (m >= M) continue;
+            float mx = -INFINITY;
+#pragma unroll
+            for (int w = 0; w < kAttnWarps; ++w) mx = fmaxf(mx, wpart[(size_t)w * 16 * (HD + 2) + rr * (HD + 2)]);
+            float out;
+            if (col == 0) {
+                out = mx;
+            } else if (mx == -INFINITY) {
+                out = 0.f;
+            } else {
+                out = 0.f;
+#pragma unroll
+                for (int w = 0; w < kAttnWarps; ++w) {
+                    const float* wpw = wpart + (size_t)w * 16 * (HD + 2) + rr * (HD + 2);
+                    const float mw = wpw[0];
+                    if (mw != -INFINITY) out += exp2f(mw - mx) * wpw[col];
+                }
+            }
+            const int r = m / G, gq = m - r * G;
+            float* dst = a.part + (((size_t)r * a.hq + h * G + gq) * a.n_chunks_max + c) * (HD + 2);
+            dst[col] = out;
+        }
+        __syncthreads();
+    }
+}
+
+// ----------------------------------------------------------- fp32 kernel
+// One warp per query row at a time; K/V read from the cache (L2).
+template <int HD>
+__global__ void __launch_bounds__(128) attn_f32_kernel(const AttnArgs a) {
+    constexpr int NPL = HD / 32;
+    constexpr int C = kAttnChunk;
+    __shared__ float qsh[kAttnWarps][HD];
+    __shared__ float psh[kAttnWarps][C];
+    const int h = blockIdx.x, c = blockIdx.y;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int G = a.hq / a.hk;
+    const int M = G * a.R;
+    const int cs = c * C;
+    const int ce = min(cs + C, a.p0 + a.R);
+
+    write_new_kv<float, NPL>(a, h, cs, ce);
+    __syncthreads();
+
+    const float* kc = reinterpret_cast<const float*>(a.kcache) + (size_t)h * a.max_seq * HD;
+    const float* vc = reinterpret_cast<const float*>(a.vcache) + (size_t)h * a.max_seq * HD;
+    const float qscale = kLog2e * rsqrtf((float)HD);
+    const float* qn = reinterpret_cast<const float*>(a.q_norm);
+    for (int m = warp; m < M; m += kAttnWarps) {
+        const int r = m / G, gq = m - r * G;
+        const int pos = a.p0 + r;
+        float q[NPL];
+        head_vector<float, NPL>(a.qkv + (size_t)r * a.qkv_ld + (h * G + gq) * HD, qn, a.eps, a.rope, pos, q);
+#pragma unroll
+        for (int i = 0; i < NPL; ++i) qsh[warp][lane + 32 * i] = q[i] * qscale;
+        __syncwarp();
+        const int kend = min(ce, pos + 1);
+        // scores: lane owns keys cs + lane + 32 j
+        float mx = -INFINITY;
+        for (int j = lane; j < C; j += 32) {
+            const int key = cs + j;
+            float sc = -INFINITY;
+            if (key < kend) {
+                sc = 0.f;
+                const float* kr = kc + (size_t)key * HD;
+                for (int d = 0; d < HD; ++d) sc = fmaf(qsh[warp][d], kr[d], sc);
+            }
+            psh[warp][j] = sc;
+            mx = fmaxf(mx, sc);
+        }
+        mx = warp_max(mx);
+        float l = 0.f;
+        for (int j = lane; j < C; j += 32) {
+            const float p = (mx == -INFINITY || psh[warp][j] == -INFINITY) ? 0.f : exp2f(psh[warp][j] - mx);
+            psh[warp][j] = p;
+            l += p;
+        }
+        l = warp_sum(l);
+        __syncwarp();
+        float* dst = a.part + (((size_t)r * a.hq + h * G + gq) * a.n_chunks_max + c) * (HD + 2);
+        for (int d = lane; d < HD; d += 32) {
+            float acc = 0.f;
+            for (int j = 0; j < kend - cs; ++j) acc = fmaf(psh[warp][j], vc[(size_t)(cs + j) * HD + d], acc);
+            dst[2 + d] = acc;
+        }
+        if (lane == 0) {
+            dst[0] = mx;
+            dst[1] = l;
+        }
+        __syncwarp();
+    }
+}
+
+// ------------------------------------------------------------------ merge
+// out[r][hq_idx * hd + d] = sum_c 2^(m_c - M) o_c[d] / sum_c 2^(m_c - M) l_c over
+// the chunks 0 .. pos_r / C of row r, in chunk order.
+template <typename WT, int HD>
+__global__ void __launch_bounds__(HD) attn_merge_kernel(const AttnArgs a) {
+    const int hq_idx = blockIdx.x, r = blockIdx.y, d = threadIdx.x;
+    const int pos = a.p0 + r;
+    const int nch = pos / kAttnChunk + 1;
+    const float* base = a.part + ((size_t)r * a.hq + hq_idx) * a.n_chunks_max * (HD + 2);
+    float mx = -INFINITY;
+    for (int c = 0; c < nch; ++c) mx = fmaxf(mx, base[(size_t)c * (HD + 2)]);
+    float L = 0.f, O = 0.f;
+    for (int c = 0; c < nch; ++c) {
+        const float* p = base + (size_t)c * (HD + 2);
+        const float m = p[0];
+        if (m == -INFINITY) continue;
+        const float w = exp2f(m - mx);
+        L += w * p[1];
+        O += w * p[2 + d];
+    }
+    WT* out = reinterpret_cast<WT*>(a.out);
+    out[(size_t)r * a.out_ld + hq_idx * HD + d] = from_float<WT>(O / L);
+}
+
+// --------------------------------------------------------------- launchers
+static size_t attn_bf16_smem(int HD, int mpad) {
+    const int P = HD + 8;
+    return sizeof(__nv_bfloat16) * ((size_t)mpad * P + 2 * (size_t)kAttnChunk * P) +
+           sizeof(float) * kAttnWarps * 16 * (HD + 2);
+}
+
+cudaError_t launch_attention(int dtype, const AttnArgs& a, cudaStream_t s) {
+    const int nch = (a.p0 + a.R + kAttnChunk - 1) / kAttnChunk;
+    if (nch > a.n_chunks_max) return cudaErrorInvalidValue;
+    dim3 grid(a.hk, nch);
+    if (dtype == 1) {
+        const int M = (a.hq / a.hk) * a.R;
+        const int mpad = ((M + 15) / 16) * 16;
+        const size_t smem = attn_bf16_smem(a.hd, mpad);
+        auto run = [&](auto kern) -> cudaError_t {
+            cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+            if (e != cudaSuccess) return e;
+            kern<<<grid, 128, smem, s>>>(a);
+            return cudaGetLastError();
+        };
+        if (a.hd == 128) return run(attn_bf16_kernel<128>);
+        if (a.hd == 64) return run(attn_bf16_kernel<64>);
+        return cudaErrorInvalidValue;
+    }
+    if (a.hd == 128) attn_f32_kernel<128><<<grid, 128, 0, s>>>(a);
+    else if (a.hd == 64) attn_f32_kernel<64><<<grid, 128, 0, s>>>(a);
+    else return cudaErrorInvalidValue;
+    return cudaGetLastError();
+}
+
+cudaError_t launch_attn_merge(int dtype, const AttnArgs& a, cudaStream_t s) {
+    dim3 grid(a.hq, a.R);
+    if (dtype == 1) {
+        if (a.hd == 128) attn_merge_kernel<__nv_bfloat16, 128><<<grid, 128, 0, s>>>(a);
+        else attn_merge_kernel<__nv_bfloat16, 64><<<grid, 64, 0, s>>>(a);
+    } else {
+        if (a.hd == 128) attn_merge_kernel<float, 128><<<grid, 128, 0, s>>>(a);
+        else attn_merge_kernel<float, 64><<<grid, 64, 0, s>>>(a);
+    }
+    return cudaGetLastError();
+}
+
+}  // namespace ks

@@ -1,0 +1,897 @@
+// Model runtime and C ABI of libknapspec: workspace layout, the skip-masked
+// forward pass (Sec. 2), draft (a1), verify + greedy acceptance (a2, a3,
+// Sec. 2.1), the history ring (Sec. 3.4), and the speculative loop that
+// re-selects the draft mask with the knapsack (a4, a5).
+//
+// All device memory is the caller's workspace; this file carves it up.  The
+// host loop launches one kernel per matrix product (5 per layer plus the
+// attention split/merge pair) on the caller's stream; draft tokens stay on
+// the device between steps and one stream synchronisation per verify step
+// returns the accepted tokens.
+#include "../../include/knapspec.h"
+#include "common.cuh"
+#include "internal.h"
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <vector>
+
+namespace ks {
+
+static thread_local char g_err[512] = "";
+
+void set_error(const char* fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_err, sizeof(g_err), fmt, ap);
+    va_end(ap);
+}
+
+size_t select_scratch_bytes(int n_items, int cap);
+cudaError_t launch_select(const ks_latency* lat, const float* sims, int64_t n, int n_items, int budget,
+                          double budget_frac, uint8_t* mask, double* objective, int32_t* weights,
+                          int32_t* budget_out, void* scratch, int cap, cudaStream_t s);
+
+constexpr int kSelectCap = 65535;
+constexpr int kKlasses = 9;
+enum { K_QKV = 0, K_ATTN, K_MERGE, K_OPROJ, K_GATEUP, K_DOWN, K_LMHEAD, K_EMBED, K_ACCEPT };
+
+// ------------------------------------------------------------ small kernels
+// x[r] = embed[tok[r]] (fp32); optionally copied to the history plane 0.
+template <typename WT>
+__global__ void embed_kernel(const WT* embed, const int32_t* tok, int d, int vocab, float* x,
+                             float* capture) {
+    const int r = blockIdx.x;
+    int t = tok[r];
+    if (t < 0 || t >= vocab) t = 0;
+    const WT* e = embed + (size_t)t * d;
+    for (int k = threadIdx.x; k < d; k += blockDim.x) {
+        const float v = to_float(e[k]);
+        x[(size_t)r * d + k] = v;
+        if (capture) capture[(size_t)r * d + k] = v;
+    }
+}
+
+// Greedy acceptance (Sec. 2.1): drafts = rows[1..gamma], z = target argmax of
+// rows[0..gamma].  a = longest prefix with drafts[i] == z[i]; the new tokens
+// are drafts[0..a-1] followed by z[a], which becomes the pending rows[0].
+// result = {a, a + 1, tokens[0..a]}.
+__global__ void accept_kernel(int32_t* rows, const int32_t* z, int gamma, int32_t* result) {
+    if (threadIdx.x != 0) return;
+    int a = 0;
+    while (a < gamma && rows[1 + a] == z[a]) ++a;
+    result[0] = a;
+    result[1] = a + 1;
+    for (int i = 0; i < a; ++i) result[2 + i] = rows[1 + i];
+    result[2 + a] = z[a];
+    rows[0] = z[a];
+}
+
+// ------------------------------------------------------------------ helpers
+static size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+struct Layout {
+    size_t kv, rope, x, qkv, attn_out, act, attn_part, gemv_part, counters, logits, amax_val,
+        amax_idx, tok, hist, hist_idx, sims, mask, obj, wts, select, total;
+    int n_chunks_max;
+    size_t gemv_part_floats;
+    int counters_n;
+    int hist_slots;
+};
+
+static bool config_ok(const ks_config* c) {
+    if (!c) return false;
+    if (c->n_layers < 1 || c->n_layers > 128) return false;
+    if (c->d_model < 8 || c->d_model % 8) return false;
+    if (c->n_q_heads < 1 || c->n_kv_heads < 1 || c->n_q_heads % c->n_kv_heads) return false;
+    if (c->n_q_heads / c->n_kv_heads > 16) return false;
+    if (c->head_dim != 64 && c->head_dim != 128) return false;
+    if (c->d_ff < 8 || c->d_ff % 8) return false;
+    if (c->vocab < 1) return false;
+    if (c->dtype != KS_DTYPE_F32 && c->dtype != KS_DTYPE_BF16) return false;
+    if (c->max_seq < 2 || c->max_rows < 2 || c->max_rows > 16) return false;
+    if (c->hist_steps < 1 || c->hist_steps > 64) return false;
+    if (c->hist_init_rows < 1 || c->hist_init_rows > c->max_rows) return false;
+    if (!(c->rms_eps > 0.f) || !(c->rope_theta > 1.0)) return false;
+    return true;
+}
+
+static Layout make_layout(const ks_config* c) {
+    Layout L{};
+    const size_t es = c->dtype == KS_DTYPE_BF16 ? 2 : 4;
+    const int d = c->d_model, hd = c->head_dim, R = c->max_rows;
+    const int nqkv = (c->n_q_heads + 2 * c->n_kv_heads) * hd;
+    const int nsub = 2 * c->n_layers;
+    L.n_chunks_max = (c->max_seq + kAttnChunk - 1) / kAttnChunk;
+    L.hist_slots = c->hist_steps + 1;
+    size_t gp = 0;
+    gp = std::max(gp, gemv_partial_floats(nqkv, d, R, EPI_STORE));
+    gp = std::max(gp, gemv_partial_floats(d, c->n_q_heads * hd, R, EPI_RESID));
+    gp = std::max(gp, gemv_partial_floats(c->d_ff, d, R, EPI_SWIGLU));
+    gp = std::max(gp, gemv_partial_floats(d, c->d_ff, R, EPI_RESID));
+    L.gemv_part_floats = gp;
+    int gx = gemv_grid_x(c->vocab);
+    gx = std::max(gx, gemv_grid_x(nqkv));
+    gx = std::max(gx, gemv_grid_x(c->d_ff));
+    gx = std::max(gx, gemv_grid_x(d));
+    L.counters_n = gx + 1;
+
+    size_t off = 0;
+    auto take = [&](size_t bytes) {
+        size_t o = off;
+        off = align_up(off + bytes, 256);
+        return o;
+    };
+    L.kv = take(2 * (size_t)c->n_layers * c->n_kv_heads * (size_t)c->max_seq * hd * es);
+    L.rope = take(sizeof(float) * (size_t)c->max_seq * hd);
+    L.x = take(sizeof(float) * (size_t)R * d);
+    L.qkv = take(sizeof(float) * (size_t)R * nqkv);
+    L.attn_out = take(es * (size_t)R * c->n_q_heads * hd);
+    L.act = take(es * (size_t)R * c->d_ff);
+    L.attn_part = take(sizeof(float) * (size_t)R * c->n_q_heads * L.n_chunks_max * (hd + 2));
+    L.gemv_part = take(sizeof(float) * std::max<size_t>(gp, 1));
+    L.counters = take(sizeof(int) * (size_t)L.counters_n);
+    L.logits = take(sizeof(float) * (size_t)R * c->vocab);
+    L.amax_val = take(sizeof(float) * (size_t)gemv_grid_x(c->vocab) * 16);
+    L.amax_idx = take(sizeof(int) * (size_t)gemv_grid_x(c->vocab) * 16);
+    // tokens: rows[R+1] | target[R] | result[R+3] | prompt/out[max_seq]
+    L.tok = take(sizeof(int) * ((size_t)3 * R + 8 + c->max_seq));
+    L.hist = take(sizeof(float) * (size_t)(nsub + 1) * L.hist_slots * R * d);
+    L.hist_idx = take(sizeof(int) * (size_t)L.hist_slots * R);
+    L.sims = take(sizeof(float) * nsub);
+    L.mask = take(nsub);
+    L.obj = take(sizeof(double) * 2);
+    L.wts = take(sizeof(int) * (nsub + 2));
+    L.select = take(select_scratch_bytes(nsub, kSelectCap));
+    L.total = off;
+    return L;
+}
+
+}  // namespace ks
+
+using namespace ks;
+
+struct KlassTiming {
+    bool on = false;
+    std::vector<cudaEvent_t> ev;  // pairs
+    size_t used = 0;
+};
+
+struct ks_model {
+    ks_config cfg;
+    int dtype;
+    size_t es;
+    int nsub;
+    const void* embed;
+    const void* lm_head;
+    const void* final_norm;
+    std::vector<const void*> attn_norm, w_qkv, w_o, q_norm, k_norm, mlp_norm, w_gate_up, w_down;
+    cudaStream_t stream;
+    char* ws;
+    size_t ws_bytes;
+    Layout lay;
+    // carved pointers
+    char* kv;
+    float *rope, *x, *qkv, *attn_part, *gemv_part, *logits, *amax_val, *hist, *sims;
+    void *attn_out, *act, *select;
+    int *counters, *amax_idx, *rows, *target, *result, *seq, *hist_idx;
+    uint8_t* mask_dev;
+    double* obj_dev;
+    int* wts_dev;
+    // pinned host staging
+    int32_t* h_buf;
+    size_t h_buf_ints;
+    // decoding state
+    bool have_seq = false;
+    int p = 0;
+    int pending = 0;
+    int last_gamma = -1;
+    int last_pass_rows = 0;
+    std::vector<int> slot_off, slot_cnt;  // history ring rows per slot
+    int hist_next = 0;
+    int64_t launches = 0;
+    int64_t h2d = 0, d2h = 0;
+    KlassTiming timing[kKlasses];
+};
+
+// ----------------------------------------------------------------- plumbing
+static ks_status cuda_fail(cudaError_t e, const char* what) {
+    set_error("%s: %s", what, cudaGetErrorString(e));
+    return KS_ERR_CUDA;
+}
+
+#define KS_CUDA(call, what)                                   \
+    do {                                                      \
+        cudaError_t e_ = (call);                              \
+        if (e_ != cudaSuccess) return cuda_fail(e_, what);    \
+    } while (0)
+
+template <class F>
+static ks_status launch(ks_model* m, int klass, F&& f, const char* what) {
+    KlassTiming& T = m->timing[klass];
+    cudaEvent_t e0 = nullptr, e1 = nullptr;
+    if (T.on) {
+        if (T.used + 2 > T.ev.size()) {
+            for (int i = 0; i < 64; ++i) {
+                cudaEvent_t e;
+                KS_CUDA(cudaEventCreate(&e), "cudaEventCreate");
+                T.ev.push_back(e);
+            }
+        }
+        e0 = T.ev[T.used];
+        e1 = T.ev[T.used + 1];
+        T.used += 2;
+        KS_CUDA(cudaEventRecord(e0, m->stream), "cudaEventRecord");
+    }
+    cudaError_t e = f();
+    if (e != cudaSuccess) return cuda_fail(e, what);
+    m->launches++;
+    if (T.on) KS_CUDA(cudaEventRecord(e1, m->stream), "cudaEventRecord");
+    return KS_OK;
+}
+
+#define KS_TRY(expr)                   \
+    do {                               \
+        ks_status s_ = (expr);         \
+        if (s_ != KS_OK) return s_;    \
+    } while (0)
+
+static float* hist_plane(ks_model* m, int plane) {
+    const size_t plane_elems = (size_t)m->lay.hist_slots * m->cfg.max_rows * m->cfg.d_model;
+    return m->hist + (size_t)plane * plane_elems;
+}
+
+static void* kcache(ks_model* m, int layer) {
+    const size_t per = (size_t)m->cfg.n_kv_heads * m->cfg.max_seq * m->cfg.head_dim * m->es;
+    return m->kv + (size_t)(2 * layer) * per;
+}
+static void* vcache(ks_model* m, int layer) {
+    const size_t per = (size_t)m->cfg.n_kv_heads * m->cfg.max_seq * m->cfg.head_dim * m->es;
+    return m->kv + (size_t)(2 * layer + 1) * per;
+}
+
+// One pass of f^(S) over R consecutive rows at positions p0..p0+R-1.
+// tok: device token ids of the rows.  mask: host uint8[2L] or null (all).
+// capture_slot >= 0: write X^(i) of every row into the history slot (all
+// sublayers must run).  argmax: device int32[R] for the LM head argmax, or
+// null to skip the LM head.
+static ks_status forward(ks_model* m, const int32_t* tok, int R, int p0, const uint8_t* mask,
+                         int capture_slot, int32_t* argmax) {
+    const ks_config& c = m->cfg;
+    const int d = c.d_model, hd = c.head_dim;
+    const int nqkv = (c.n_q_heads + 2 * c.n_kv_heads) * hd;
+    const int dt = m->dtype;
+    cudaStream_t s = m->stream;
+    auto cap_ptr = [&](int plane) -> float* {
+        if (capture_slot < 0) return nullptr;
+        return hist_plane(m, plane) + (size_t)capture_slot * c.max_rows * d;
+    };
+    KS_TRY(launch(m, K_EMBED, [&]() -> cudaError_t {
+        if (dt == KS_DTYPE_BF16)
+            embed_kernel<__nv_bfloat16><<<R, 256, 0, s>>>(reinterpret_cast<const __nv_bfloat16*>(m->embed), tok, d,
+                                                           c.vocab, m->x, cap_ptr(0));
+        else
+            embed_kernel<float><<<R, 256, 0, s>>>(reinterpret_cast<const float*>(m->embed), tok, d, c.vocab, m->x,
+                                                  cap_ptr(0));
+        return cudaGetLastError();
+    }, "embed"));
+
+    for (int l = 0; l < c.n_layers; ++l) {
+        const bool run_attn = !mask || mask[2 * l];
+        const bool run_mlp = !mask || mask[2 * l + 1];
+        if (run_attn) {
+            GemvArgs g{};
+            g.W = m->w_qkv[l]; g.N = nqkv; g.K = d; g.R = R;
+            g.in = m->x; g.in_ld = d; g.norm_gain = m->attn_norm[l]; g.eps = c.rms_eps;
+            g.out = m->qkv; g.out_ld = nqkv;
+            g.partial = m->gemv_part; g.counters = m->counters;
+            gemv_plan(g, EPI_STORE);
+            KS_TRY(launch(m, K_QKV, [&] { return launch_gemv(dt, EPI_STORE, g, s); }, "qkv"));
+
+            AttnArgs at{};
+            at.qkv = m->qkv; at.qkv_ld = nqkv; at.R = R; at.p0 = p0;
+            at.hq = c.n_q_heads; at.hk = c.n_kv_heads; at.hd = hd;
+            at.kcache = kcache(m, l); at.vcache = vcache(m, l); at.max_seq = c.max_seq;
+            at.rope = m->rope;
+            at.q_norm = c.qk_norm ? m->q_norm[l] : nullptr;
+            at.k_norm = c.qk_norm ? m->k_norm[l] : nullptr;
+            at.eps = c.rms_eps; at.chunk = kAttnChunk;
+            at.part = m->attn_part; at.n_chunks_max = m->lay.n_chunks_max;
+            at.out = m->attn_out; at.out_ld = c.n_q_heads * hd;
+            KS_TRY(launch(m, K_ATTN, [&] { return launch_attention(dt, at, s); }, "attention"));
+            KS_TRY(launch(m, K_MERGE, [&] { return launch_attn_merge(dt, at, s); }, "attention merge"));
+
+            GemvArgs o{};
+            o.W = m->w_o[l]; o.N = d; o.K = c.n_q_heads * hd; o.R = R;
+            o.in = m->attn_out; o.in_ld = c.n_q_heads * hd;
+            o.resid = m->x; o.resid_ld = d;
+            o.capture = cap_ptr(2 * l + 1); o.capture_ld = d;
+            o.partial = m->gemv_part; o.counters = m->counters;
+            gemv_plan(o, EPI_RESID);
+            KS_TRY(launch(m, K_OPROJ, [&] { return launch_gemv(dt, EPI_RESID, o, s); }, "o-proj"));
+        } else if (capture_slot >= 0) {
+            set_error("forward: capture needs every sublayer");
+            return KS_ERR_STATE;
+        }
+        if (run_mlp) {
+            GemvArgs gu{};
+            gu.W = m->w_gate_up[l]; gu.N = c.d_ff; gu.K = d; gu.R = R;
+            gu.in = m->x; gu.in_ld = d; gu.norm_gain = m->mlp_norm[l]; gu.eps = c.rms_eps;
+            gu.act = m->act; gu.act_ld = c.d_ff;
+            gu.partial = m->gemv_part; gu.counters = m->counters;
+            gemv_plan(gu, EPI_SWIGLU);
+            KS_TRY(launch(m, K_GATEUP, [&] { return launch_gemv(dt, EPI_SWIGLU, gu, s); }, "gate-up"));
+
+            GemvArgs dn{};
+            dn.W = m->w_down[l]; dn.N = d; dn.K = c.d_ff; dn.R = R;
+            dn.in = m->act; dn.in_ld = c.d_ff;
+            dn.resid = m->x; dn.resid_ld = d;
+            dn.capture = cap_ptr(2 * l + 2); dn.capture_ld = d;
+            dn.partial = m->gemv_part; dn.counters = m->counters;
+            gemv_plan(dn, EPI_RESID);
+            KS_TRY(launch(m, K_DOWN, [&] { return launch_gemv(dt, EPI_RESID, dn, s); }, "down"));
+        } else if (capture_slot >= 0) {
+            set_error("forward: capture needs every sublayer");
+            return KS_ERR_STATE;
+        }
+    }
+    if (argmax) {
+        GemvArgs lm{};
+        lm.W = m->lm_head; lm.N = c.vocab; lm.K = d; lm.R = R;
+        lm.in = m->x; lm.in_ld = d; lm.norm_gain = m->final_norm; lm.eps = c.rms_eps;
+        lm.logits = m->logits; lm.logits_ld = c.vocab;
+        lm.amax_val = m->amax_val; lm.amax_idx = m->amax_idx; lm.tokens = argmax;
+        lm.counters = m->counters;
+        gemv_plan(lm, EPI_LMHEAD);
+        KS_TRY(launch(m, K_LMHEAD, [&] { return launch_gemv(dt, EPI_LMHEAD, lm, s); }, "lm-head"));
+    }
+    m->last_pass_rows = R;
+    return KS_OK;
+}
+
+static ks_status sync(ks_model* m, const char* what) {
+    cudaError_t e = cudaStreamSynchronize(m->stream);
+    if (e != cudaSuccess) return cuda_fail(e, what);
+    return KS_OK;
+}
+
+// ------------------------------------------------------------------- C ABI
+extern "C" {
+
+const char* ks_status_str(ks_status s) {
+    switch (s) {
+        case KS_OK: return "KS_OK";
+        case KS_ERR_INVALID_ARG: return "KS_ERR_INVALID_ARG";
+        case KS_ERR_CUDA: return "KS_ERR_CUDA";
+        case KS_ERR_WORKSPACE: return "KS_ERR_WORKSPACE";
+        case KS_ERR_CAPACITY: return "KS_ERR_CAPACITY";
+        case KS_ERR_TIMEOUT: return "KS_ERR_TIMEOUT";
+        case KS_ERR_UNSUPPORTED: return "KS_ERR_UNSUPPORTED";
+        case KS_ERR_STATE: return "KS_ERR_STATE";
+    }
+    return "KS_ERR_UNKNOWN";
+}
+
+const char* ks_last_error(void) { return g_err; }
+
+size_t ks_workspace_bytes(const ks_config* cfg) {
+    if (!config_ok(cfg)) return 0;
+    return make_layout(cfg).total;
+}
+
+ks_status ks_model_create(const ks_config* cfg, const ks_weights* w, void* workspace, size_t workspace_bytes,
+                          void* stream, ks_model** out) {
+    if (!out) {
+        set_error("ks_model_create: out is null");
+        return KS_ERR_INVALID_ARG;
+    }
+    *out = nullptr;
+    if (!config_ok(cfg)) {
+        set_error("ks_model_create: invalid or unsupported config");
+        return KS_ERR_INVALID_ARG;
+    }
+    if (!w || !workspace) {
+        set_error("ks_model_create: null weights or workspace");
+        return KS_ERR_INVALID_ARG;
+    }
+    if (reinterpret_cast<uintptr_t>(workspace) & 255) {
+        set_error("ks_model_create: workspace must be 256-byte aligned");
+        return KS_ERR_INVALID_ARG;
+    }
+    const Layout lay = make_layout(cfg);
+    if (workspace_bytes < lay.total) {
+        set_error("ks_model_create: workspace %zu < required %zu", workspace_bytes, lay.total);
+        return KS_ERR_WORKSPACE;
+    }
+    const int L = cfg->n_layers;
+    auto aligned = [](const void* p) { return p && (reinterpret_cast<uintptr_t>(p) & 15) == 0; };
+    if (!aligned(w->embed) || !aligned(w->lm_head) || !aligned(w->final_norm) || !w->attn_norm || !w->w_qkv ||
+        !w->w_o || !w->mlp_norm || !w->w_gate_up || !w->w_down || (cfg->qk_norm && (!w->q_norm || !w->k_norm))) {
+        set_error("ks_model_create: missing or misaligned weight pointer");
+        return KS_ERR_INVALID_ARG;
+    }
+    for (int l = 0; l < L; ++l) {
+        if (!aligned(w->attn_norm[l]) || !aligned(w->w_qkv[l]) || !aligned(w->w_o[l]) || !aligned(w->mlp_norm[l]) ||
+            !aligned(w->w_gate_up[l]) || !aligned(w->w_down[l]) ||
+            (cfg->qk_norm && (!aligned(w->q_norm[l]) || !aligned(w->k_norm[l])))) {
+            set_error("ks_model_create: layer %d weight pointer missing or not 16-byte aligned", l);
+            return KS_ERR_INVALID_ARG;
+        }
+    }
+    ks_model* m = new ks_model();
+    m->cfg = *cfg;
+    m->dtype = cfg->dtype;
+    m->es = cfg->dtype == KS_DTYPE_BF16 ? 2 : 4;
+    m->nsub = 2 * L;
+    m->embed = w->embed;
+    m->lm_head = w->lm_head;
+    m->final_norm = w->final_norm;
+    for (int l = 0; l < L; ++l) {
+        m->attn_norm.push_back(w->attn_norm[l]);
+        m->w_qkv.push_back(w->w_qkv[l]);
+        m->w_o.push_back(w->w_o[l]);
+        m->q_norm.push_back(cfg->qk_norm ? w->q_norm[l] : nullptr);
+        m->k_norm.push_back(cfg->qk_norm ? w->k_norm[l] : nullptr);
+        m->mlp_norm.push_back(w->mlp_norm[l]);
+        m->w_gate_up.push_back(w->w_gate_up[l]);
+        m->w_down.push_back(w->w_down[l]);
+    }
+    m->stream = reinterpret_cast<cudaStream_t>(stream);
+    m->ws = reinterpret_cast<char*>(workspace);
+    m->ws_bytes = workspace_bytes;
+    m->lay = lay;
+    char* b = m->ws;
+    m->kv = b + lay.kv;
+    m->rope = reinterpret_cast<float*>(b + lay.rope);
+    m->x = reinterpret_cast<float*>(b + lay.x);
+    m->qkv = reinterpret_cast<float*>(b + lay.qkv);
+    m->attn_out = b + lay.attn_out;
+    m->act = b + lay.act;
+    m->attn_part = reinterpret_cast<float*>(b + lay.attn_part);
+    m->gemv_part = reinterpret_cast<float*>(b + lay.gemv_part);
+    m->counters = reinterpret_cast<int*>(b + lay.counters);
+    m->logits = reinterpret_cast<float*>(b + lay.logits);
+    m->amax_val = reinterpret_cast<float*>(b + lay.amax_val);
+    m->amax_idx = reinterpret_cast<int*>(b + lay.amax_idx);
+    int* tok = reinterpret_cast<int*>(b + lay.tok);
+    const int R = cfg->max_rows;
+    m->rows = tok;
+    m->target = tok + (R + 1);
+    m->result = tok + (2 * R + 1);
+    m->seq = tok + (3 * R + 8);
+    m->hist = reinterpret_cast<float*>(b + lay.hist);
+    m->hist_idx = reinterpret_cast<int*>(b + lay.hist_idx);
+    m->sims = reinterpret_cast<float*>(b + lay.sims);
+    m->mask_dev = reinterpret_cast<uint8_t*>(b + lay.mask);
+    m->obj_dev = reinterpret_cast<double*>(b + lay.obj);
+    m->wts_dev = reinterpret_cast<int*>(b + lay.wts);
+    m->select = b + lay.select;
+    m->slot_off.assign(lay.hist_slots, 0);
+    m->slot_cnt.assign(lay.hist_slots, 0);
+
+    auto fail = [&](cudaError_t e, const char* what) {
+        ks_status st = cuda_fail(e, what);
+        if (m->h_buf) cudaFreeHost(m->h_buf);
+        delete m;
+        return st;
+    };
+    m->h_buf_ints = (size_t)cfg->max_seq + 4 * (size_t)R + 64 + lay.hist_slots * (size_t)R + 2 * (size_t)L + 64;
+    cudaError_t e = cudaHostAlloc(reinterpret_cast<void**>(&m->h_buf), m->h_buf_ints * sizeof(int32_t),
+                                  cudaHostAllocDefault);
+    if (e != cudaSuccess) {
+        m->h_buf = nullptr;
+        return fail(e, "cudaHostAlloc");
+    }
+    // RoPE table in double, rounded to fp32: [pos][j][cos, sin]
+    {
+        const int hd = cfg->head_dim, half = hd / 2;
+        std::vector<float> tab((size_t)cfg->max_seq * hd);
+        std::vector<double> inv(half);
+        for (int j = 0; j < half; ++j) inv[j] = std::pow(cfg->rope_theta, -2.0 * j / hd);
+        for (int p = 0; p < cfg->max_seq; ++p)
+            for (int j = 0; j < half; ++j) {
+                const double ang = (double)p * inv[j];
+                tab[((size_t)p * half + j) * 2] = (float)std::cos(ang);
+                tab[((size_t)p * half + j) * 2 + 1] = (float)std::sin(ang);
+            }
+        e = cudaMemcpyAsync(m->rope, tab.data(), tab.size() * sizeof(float), cudaMemcpyHostToDevice, m->stream);
+        if (e != cudaSuccess) return fail(e, "rope upload");
+        e = cudaStreamSynchronize(m->stream);
+        if (e != cudaSuccess) return fail(e, "rope upload");
+    }
+    e = cudaMemsetAsync(m->counters, 0, sizeof(int) * lay.counters_n, m->stream);
+    if (e != cudaSuccess) return fail(e, "counter reset");
+    e = cudaMemsetAsync(b + lay.tok, 0, sizeof(int) * ((size_t)3 * R + 8 + cfg->max_seq), m->stream);
+    if (e != cudaSuccess) return fail(e, "token reset");
+    e = cudaStreamSynchronize(m->stream);
+    if (e != cudaSuccess) return fail(e, "create sync");
+    *out = m;
+    return KS_OK;
+}
+
+ks_status ks_model_destroy(ks_model* m) {
+    if (!m) return KS_ERR_INVALID_ARG;
+    cudaStreamSynchronize(m->stream);
+    for (auto& T : m->timing)
+        for (auto e : T.ev) cudaEventDestroy(e);
+    if (m->h_buf) cudaFreeHost(m->h_buf);
+    delete m;
+    return KS_OK;
+}
+
+ks_status ks_prefill(ks_model* m, const int32_t* tokens, int32_t n, int32_t* next_token) {
+    if (!m || !tokens || !next_token) {
+        set_error("ks_prefill: null argument");
+        return KS_ERR_INVALID_ARG;
+    }
+    const ks_config& c = m->cfg;
+    if (n < 1) {
+        set_error("ks_prefill: n must be >= 1");
+        return KS_ERR_INVALID_ARG;
+    }
+    if (n + 1 > c.max_seq) {
+        set_error("ks_prefill: prompt of %d does not fit max_seq %d", n, c.max_seq);
+        return KS_ERR_CAPACITY;
+    }
+    for (int i = 0; i < n; ++i)
+        if (tokens[i] < 0 || tokens[i] >= c.vocab) {
+            set_error("ks_prefill: token %d out of range", i);
+            return KS_ERR_INVALID_ARG;
+        }
+    m->have_seq = false;
+    std::memcpy(m->h_buf, tokens, sizeof(int32_t) * n);
+    KS_CUDA(cudaMemcpyAsync(m->seq, m->h_buf, sizeof(int32_t) * n, cudaMemcpyHostToDevice, m->stream), "prompt upload");
+    m->h2d += sizeof(int32_t) * n;
+    const int R = c.max_rows;
+    // chunks aligned to the end so the last chunk holds the last R rows
+    const int first = n - R * ((n - 1) / R);
+    int start = 0;
+    int len = first;
+    const int init_slot = 0;
+    while (start < n) {
+        const bool last = (start + len == n);
+        KS_TRY(forward(m, m->seq + start, len, start, nullptr, last ? init_slot : -1, last ? m->target : nullptr));
+        start += len;
+        len = R;
+    }
+    // pending = argmax of the last prompt row
+    const int lastlen = (n <= R) ? n : R;
+    KS_CUDA(cudaMemcpyAsync(m->rows, m->target + (lastlen - 1), sizeof(int32_t), cudaMemcpyDeviceToDevice, m->stream),
+            "pending");
+    KS_CUDA(cudaMemcpyAsync(m->h_buf, m->rows, sizeof(int32_t), cudaMemcpyDeviceToHost, m->stream), "pending");
+    m->d2h += sizeof(int32_t);
+    KS_TRY(sync(m, "ks_prefill"));
+    m->pending = m->h_buf[0];
+    *next_token = m->pending;
+    m->p = n;
+    m->have_seq = true;
+    m->last_gamma = -1;
+    std::fill(m->slot_cnt.begin(), m->slot_cnt.end(), 0);
+    const int init = std::min(c.hist_init_rows, lastlen);
+    m->slot_off[init_slot] = lastlen - init;
+    m->slot_cnt[init_slot] = init;
+    m->hist_next = 1;
+    return KS_OK;
+}
+
+ks_status ks_draft(ks_model* m, const uint8_t* mask, int32_t gamma, int32_t* draft_tokens) {
+    if (!m || !mask) {
+        set_error("ks_draft: null argument");
+        return KS_ERR_INVALID_ARG;
+    }
+    if (!m->have_seq) {
+        set_error("ks_draft: no sequence (call ks_prefill first)");
+        return KS_ERR_STATE;
+    }
+    if (gamma < 1 || gamma >= m->cfg.max_rows) {
+        set_error("ks_draft: gamma must be in [1, max_rows)");
+        return KS_ERR_INVALID_ARG;
+    }
+    if (m->p + gamma + 1 > m->cfg.max_seq) {
+        set_error("ks_draft: KV capacity exceeded");
+        return KS_ERR_CAPACITY;
+    }
+    for (int t = 0; t < gamma; ++t)
+        KS_TRY(forward(m, m->rows + t, 1, m->p + t, mask, -1, m->rows + t + 1));
+    m->last_gamma = gamma;
+    if (draft_tokens) {
+        KS_CUDA(cudaMemcpyAsync(m->h_buf, m->rows + 1, sizeof(int32_t) * gamma, cudaMemcpyDeviceToHost, m->stream),
+                "draft download");
+        m->d2h += sizeof(int32_t) * gamma;
+        KS_TRY(sync(m, "ks_draft"));
+        std::memcpy(draft_tokens, m->h_buf, sizeof(int32_t) * gamma);
+    }
+    return KS_OK;
+}
+
+ks_status ks_verify(ks_model* m, const int32_t* draft_tokens, int32_t gamma, int32_t* n_accepted,
+                    int32_t* out_tokens, int32_t* n_out) {
+    if (!m || !n_accepted || !out_tokens || !n_out) {
+        set_error("ks_verify: null argument");
+        return KS_ERR_INVALID_ARG;
+    }
+    if (!m->have_seq) {
+        set_error("ks_verify: no sequence (call ks_prefill first)");
+        return KS_ERR_STATE;
+    }
+    if (gamma < 1 || gamma >= m->cfg.max_rows) {
+        set_error("ks_verify: gamma must be in [1, max_rows)");
+        return KS_ERR_INVALID_ARG;
+    }
+    if (m->p + gamma + 1 > m->cfg.max_seq) {
+        set_error("ks_verify: KV capacity exceeded");
+        return KS_ERR_CAPACITY;
+    }
+    if (draft_tokens) {
+        for (int i = 0; i < gamma; ++i)
+            if (draft_tokens[i] < 0 || draft_tokens[i] >= m->cfg.vocab) {
+                set_error("ks_verify: draft token %d out of range", i);
+                return KS_ERR_INVALID_ARG;
+            }
+        int32_t* hb = m->h_buf + m->cfg.max_seq;  // separate staging region
+        std::memcpy(hb, draft_tokens, sizeof(int32_t) * gamma);
+        KS_CUDA(cudaMemcpyAsync(m->rows + 1, hb, sizeof(int32_t) * gamma, cudaMemcpyHostToDevice, m->stream),
+                "draft upload");
+        m->h2d += sizeof(int32_t) * gamma;
+    } else if (m->last_gamma != gamma) {
+        set_error("ks_verify: no preceding ks_draft with this gamma");
+        return KS_ERR_STATE;
+    }
+    const int R = gamma + 1;
+    const int slot = m->hist_next;
+    KS_TRY(forward(m, m->rows, R, m->p, nullptr, slot, m->target));
+    KS_TRY(launch(m, K_ACCEPT, [&]() -> cudaError_t {
+        accept_kernel<<<1, 32, 0, m->stream>>>(m->rows, m->target, gamma, m->result);
+        return cudaGetLastError();
+    }, "accept"));
+    int32_t* hb = m->h_buf + m->cfg.max_seq + 2 * m->cfg.max_rows;
+    KS_CUDA(cudaMemcpyAsync(hb, m->result, sizeof(int32_t) * (gamma + 3), cudaMemcpyDeviceToHost, m->stream),
+            "result download");
+    m->d2h += sizeof(int32_t) * (gamma + 3);
+    KS_TRY(sync(m, "ks_verify"));
+    const int a = hb[0];
+    if (a < 0 || a > gamma) {
+        set_error("ks_verify: corrupt acceptance result");
+        return KS_ERR_CUDA;
+    }
+    *n_accepted = a;
+    *n_out = a + 1;
+    for (int i = 0; i <= a; ++i) out_tokens[i] = hb[2 + i];
+    m->pending = hb[2 + a];
+    m->p += a + 1;
+    m->slot_off[slot] = 0;
+    m->slot_cnt[slot] = a + 1;
+    m->hist_next = (slot + 1) % m->lay.hist_slots;
+    // keep hist_steps entries: drop the entry the next verify will overwrite
+    m->slot_cnt[m->hist_next] = 0;
+    m->last_gamma = -1;
+    return KS_OK;
+}
+
+ks_status ks_decode_greedy(ks_model* m, int32_t n_tokens, int32_t* out) {
+    if (!m || !out || n_tokens < 1) {
+        set_error("ks_decode_greedy: bad argument");
+        return KS_ERR_INVALID_ARG;
+    }
+    if (!m->have_seq) {
+        set_error("ks_decode_greedy: no sequence (call ks_prefill first)");
+        return KS_ERR_STATE;
+    }
+    if (m->p + n_tokens > m->cfg.max_seq) {
+        set_error("ks_decode_greedy: KV capacity exceeded");
+        return KS_ERR_CAPACITY;
+    }
+    // seq[0] = pending; step i feeds seq[i] at p + i and writes seq[i + 1]
+    KS_CUDA(cudaMemcpyAsync(m->seq, m->rows, sizeof(int32_t), cudaMemcpyDeviceToDevice, m->stream), "pending");
+    for (int i = 0; i + 1 < n_tokens; ++i) KS_TRY(forward(m, m->seq + i, 1, m->p + i, nullptr, -1, m->seq + i + 1));
+    KS_CUDA(cudaMemcpyAsync(m->rows, m->seq + (n_tokens - 1), sizeof(int32_t), cudaMemcpyDeviceToDevice, m->stream),
+            "pending");
+    KS_CUDA(cudaMemcpyAsync(m->h_buf, m->seq, sizeof(int32_t) * n_tokens, cudaMemcpyDeviceToHost, m->stream),
+            "tokens download");
+    m->d2h += sizeof(int32_t) * n_tokens;
+    KS_TRY(sync(m, "ks_decode_greedy"));
+    std::memcpy(out, m->h_buf, sizeof(int32_t) * n_tokens);
+    m->p += n_tokens - 1;
+    m->pending = out[n_tokens - 1];
+    m->last_gamma = -1;
+    return KS_OK;
+}
+
+ks_status ks_model_position(const ks_model* m, int32_t* committed, int32_t* pending) {
+    if (!m || !committed || !pending) return KS_ERR_INVALID_ARG;
+    *committed = m->p;
+    *pending = m->pending;
+    return KS_OK;
+}
+
+static int history_rows(ks_model* m, int32_t* idx) {
+    int r = 0;
+    const int R = m->cfg.max_rows;
+    // oldest slot first: the slot after hist_next-1 going around the ring
+    for (int k = 1; k <= m->lay.hist_slots; ++k) {
+        const int s = (m->hist_next + k) % m->lay.hist_slots;
+        for (int i = 0; i < m->slot_cnt[s]; ++i) idx[r++] = s * R + m->slot_off[s] + i;
+    }
+    return r;
+}
+
+ks_status ks_history_similarities(ks_model* m, float* sims, int32_t* rows_used) {
+    if (!m || !sims) {
+        set_error("ks_history_similarities: null argument");
+        return KS_ERR_INVALID_ARG;
+    }
+    if (!m->have_seq) {
+        set_error("ks_history_similarities: no sequence");
+        return KS_ERR_STATE;
+    }
+    int32_t* hidx = m->h_buf + m->cfg.max_seq + 4 * m->cfg.max_rows + 16;
+    const int r = history_rows(m, hidx);
+    if (r < 1) {
+        set_error("ks_history_similarities: empty history");
+        return KS_ERR_STATE;
+    }
+    KS_CUDA(cudaMemcpyAsync(m->hist_idx, hidx, sizeof(int32_t) * r, cudaMemcpyHostToDevice, m->stream),
+            "history index upload");
+    m->h2d += sizeof(int32_t) * r;
+    const int d = m->cfg.d_model;
+    const int64_t plane = (int64_t)m->lay.hist_slots * m->cfg.max_rows * d;
+    cudaError_t e = launch_cosine(hist_plane(m, 0), hist_plane(m, 1), KS_DTYPE_F32, m->nsub, r, d, plane,
+                                  m->hist_idx, sims, m->stream);
+    if (e != cudaSuccess) return cuda_fail(e, "history cosine");
+    m->launches++;
+    if (rows_used) *rows_used = r;
+    return KS_OK;
+}
+
+ks_status ks_generate_speculative(ks_model* m, const ks_spec_params* prm, int32_t n_tokens, int32_t* out,
+                                  ks_spec_stats* stats, int32_t* accepted_per_step) {
+    if (!m || !prm || !out || n_tokens < 1) {
+        set_error("ks_generate_speculative: bad argument");
+        return KS_ERR_INVALID_ARG;
+    }
+    if (!m->have_seq) {
+        set_error("ks_generate_speculative: no sequence (call ks_prefill first)");
+        return KS_ERR_STATE;
+    }
+    const int nsub = m->nsub;
+    if (prm->gamma < 1 || prm->gamma >= m->cfg.max_rows || (prm->policy != 0 && prm->policy != 1) ||
+        (prm->policy == 0 && !prm->mask) ||
+        (prm->policy == 1 && (prm->resolve_every < 1 || !(prm->budget_frac >= 0.0) || prm->budget_frac > 1.0))) {
+        set_error("ks_generate_speculative: bad parameters");
+        return KS_ERR_INVALID_ARG;
+    }
+    if (prm->policy == 1) {
+        const ks_latency& lat = prm->latency;
+        bool ok = lat.kind == 0 ? (lat.c1 > 0 && lat.c2 >= 0 && lat.c3 >= 0) : (lat.kind == 1 && lat.units);
+        if (ok && lat.kind == 1)
+            for (int i = 0; i < nsub; ++i) ok = ok && lat.units[i] >= 1 && lat.units[i] <= 65535;
+        if (!ok) {
+            set_error("ks_generate_speculative: bad latency model");
+            return KS_ERR_INVALID_ARG;
+        }
+    }
+    ks_spec_stats st{};
+    std::vector<uint8_t> mask(nsub, 1);
+    if (prm->policy == 0) std::memcpy(mask.data(), prm->mask, nsub);
+    int n = 0;
+    out[n++] = m->pending;
+    std::vector<int32_t> toks(m->cfg.max_rows + 1);
+    while (n < n_tokens && (prm->max_steps <= 0 || st.steps < prm->max_steps)) {
+        if (prm->policy == 1 && st.steps % prm->resolve_every == 0) {
+            KS_TRY(ks_history_similarities(m, m->sims, nullptr));
+            KS_TRY(launch(m, K_ACCEPT, [&] {
+                return launch_select(&prm->latency, m->sims, m->p, nsub, 0, prm->budget_frac, m->mask_dev, m->obj_dev,
+                                     m->wts_dev, m->wts_dev + nsub, m->select, kSelectCap, m->stream);
+            }, "select"));
+            uint8_t* hm = reinterpret_cast<uint8_t*>(m->h_buf + m->cfg.max_seq + 4 * m->cfg.max_rows + 16 +
+                                                     m->lay.hist_slots * m->cfg.max_rows);
+            KS_CUDA(cudaMemcpyAsync(hm, m->mask_dev, nsub, cudaMemcpyDeviceToHost, m->stream), "mask download");
+            m->d2h += nsub;
+            KS_TRY(sync(m, "select"));
+            std::memcpy(mask.data(), hm, nsub);
+            st.resolves++;
+        }
+        int g = prm->gamma;
+        if (m->p + g + 1 > m->cfg.max_seq) g = m->cfg.max_seq - m->p - 1;
+        if (g < 1) {
+            set_error("ks_generate_speculative: KV capacity exhausted");
+            return KS_ERR_CAPACITY;
+        }
+        KS_TRY(ks_draft(m, mask.data(), g, nullptr));
+        int32_t a = 0, no = 0;
+        KS_TRY(ks_verify(m, nullptr, g, &a, toks.data(), &no));
+        if (accepted_per_step) accepted_per_step[st.steps] = a;
+        st.steps++;
+        st.drafted += g;
+        st.accepted += a;
+        for (int i = 0; i < no && n < n_tokens; ++i) out[n++] = toks[i];
+    }
+    int na = 0, nm = 0;
+    for (int i = 0; i < nsub; ++i)
+        if (!mask[i]) (i % 2 == 0 ? na : nm)++;
+    st.attn_skipped = na;
+    st.mlp_skipped = nm;
+    if (stats) *stats = st;
+    return KS_OK;
+}
+
+ks_status ks_debug_read(ks_model* m, int32_t what, int32_t layer, int32_t start, int32_t count, void* dst,
+                        size_t bytes) {
+    if (!m || !dst) return KS_ERR_INVALID_ARG;
+    const ks_config& c = m->cfg;
+    cudaStream_t s = m->stream;
+    KS_TRY(sync(m, "debug sync"));
+    if (what == 0 || what == 1) {
+        const size_t row = what == 0 ? (size_t)c.vocab : (size_t)c.d_model;
+        if (count < 1 || count > c.max_rows || bytes < row * count * sizeof(float)) return KS_ERR_INVALID_ARG;
+        KS_CUDA(cudaMemcpy(dst, what == 0 ? m->logits : m->x, row * count * sizeof(float), cudaMemcpyDeviceToHost),
+                "debug read");
+        return KS_OK;
+    }
+    if (what == 2 || what == 3) {
+        if (layer < 0 || layer >= c.n_layers || start < 0 || count < 1 || start + count > c.max_seq) return KS_ERR_INVALID_ARG;
+        const size_t rowb = (size_t)c.head_dim * m->es;
+        if (bytes < rowb * count * c.n_kv_heads) return KS_ERR_INVALID_ARG;
+        const char* base = reinterpret_cast<const char*>(what == 2 ? kcache(m, layer) : vcache(m, layer));
+        KS_CUDA(cudaMemcpy2DAsync(dst, rowb * count, base + (size_t)start * rowb, rowb * c.max_seq, rowb * count,
+                                  c.n_kv_heads, cudaMemcpyDeviceToHost, s),
+                "debug kv read");
+        return sync(m, "debug kv read");
+    }
+    if (what == 4) {
+        std::vector<int32_t> idx(m->lay.hist_slots * c.max_rows);
+        const int r = history_rows(m, idx.data());
+        if (count == 0) {  // query the row count
+            if (bytes < sizeof(int32_t)) return KS_ERR_INVALID_ARG;
+            *reinterpret_cast<int32_t*>(dst) = r;
+            return KS_OK;
+        }
+        if (count != r) return KS_ERR_INVALID_ARG;
+        const size_t need = sizeof(float) * (size_t)(m->nsub + 1) * r * c.d_model;
+        if (bytes < need) return KS_ERR_INVALID_ARG;
+        float* o = reinterpret_cast<float*>(dst);
+        for (int pl = 0; pl <= m->nsub; ++pl)
+            for (int i = 0; i < r; ++i)
+                KS_CUDA(cudaMemcpy(o + ((size_t)pl * r + i) * c.d_model, hist_plane(m, pl) + (size_t)idx[i] * c.d_model,
+                                   sizeof(float) * c.d_model, cudaMemcpyDeviceToHost),
+                        "debug history read");
+        return KS_OK;
+    }
+    return KS_ERR_INVALID_ARG;
+}
+
+ks_status ks_kernel_timing(ks_model* m, int32_t klass, int32_t enable) {
+    if (!m || klass < 0 || klass >= kKlasses) return KS_ERR_INVALID_ARG;
+    KS_TRY(sync(m, "timing"));
+    m->timing[klass].on = enable != 0;
+    m->timing[klass].used = 0;
+    return KS_OK;
+}
+
+ks_status ks_kernel_time(ks_model* m, int32_t klass, int64_t* launches, double* total_ms) {
+    if (!m || klass < 0 || klass >= kKlasses || !launches || !total_ms) return KS_ERR_INVALID_ARG;
+    KS_TRY(sync(m, "timing"));
+    KlassTiming& T = m->timing[klass];
+    double tot = 0.0;
+    for (size_t i = 0; i < T.used; i += 2) {
+        float ms = 0.f;
+        KS_CUDA(cudaEventElapsedTime(&ms, T.ev[i], T.ev[i + 1]), "cudaEventElapsedTime");
+        tot += ms;
+    }
+    *launches = (int64_t)(T.used / 2);
+    *total_ms = tot;
+    return KS_OK;
+}
+
+int64_t ks_launch_count(const ks_model* m) { return m ? m->launches : -1; }
+
+ks_status ks_transfer_bytes(const ks_model* m, int64_t* h2d, int64_t* d2h) {
+    if (!m || !h2d || !d2h) return KS_ERR_INVALID_ARG;
+    *h2d = m->h2d;
+    *d2h = m->d2h;
+    return KS_OK;
+}
+
+}  // extern "C"

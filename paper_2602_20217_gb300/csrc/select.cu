@@ -1,0 +1,285 @@
+// a4 and a5 of the hot path: history cosines and knapsack mask selection.
+//
+// ks_cosine  - Sec. 2's matrix cosine, one CTA per pair; each warp takes rows
+//              in turn, the row terms are summed in row order by one thread.
+// ks_select_mask - Sec. 3.4 integer weight normalisation (App. C latency
+//              model) and the exact 0/1 knapsack of Sec. 3.3 over the 2L
+//              sublayers: items processed in order 1..2L, all capacities of
+//              an item in parallel across the CTA, int64 fixed-point values,
+//              an item taken only on strict improvement, then a backtrack
+//              from item 2L that returns the optimal mask with the smallest
+//              bitmask value.  One CTA: the table is 2L x (B + 1) with B a few
+//              hundred units, so the solve is a few microseconds.
+#include "../../include/knapspec.h"
+#include "common.cuh"
+#include "internal.h"
+
+#include <cmath>
+
+namespace ks {
+
+constexpr int kCosThreads = 256;
+
+template <typename T>
+__global__ void __launch_bounds__(kCosThreads) cosine_kernel(const T* X, const T* Y, int rows, int d,
+                                                             int64_t pair_stride, const int32_t* row_index,
+                                                             float* out) {
+    extern __shared__ float rowcos[];
+    const int p = blockIdx.x;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const T* Xp = X + (size_t)p * pair_stride;
+    const T* Yp = Y + (size_t)p * pair_stride;
+    for (int i = warp; i < rows; i += kCosThreads / 32) {
+        const int64_t ri = row_index ? row_index[i] : i;
+        const T* x = Xp + ri * d;
+        const T* y = Yp + ri * d;
+        float xy = 0.f, xx = 0.f, yy = 0.f;
+        for (int k = lane; k < d; k += 32) {
+            const float a = to_float(x[k]), b = to_float(y[k]);
+            xy = fmaf(a, b, xy);
+            xx = fmaf(a, a, xx);
+            yy = fmaf(b, b, yy);
+        }
+        xy = warp_sum(xy);
+        xx = warp_sum(xx);
+        yy = warp_sum(yy);
+        if (lane == 0) rowcos[i] = xy / (sqrtf(xx) * sqrtf(yy));
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        float s = 0.f;
+        for (int i = 0; i < rows; ++i) s += rowcos[i];
+        out[p] = s / (float)rows;
+    }
+}
+
+cudaError_t launch_cosine(const void* X, const void* Y, int dtype, int64_t n_pairs, int rows, int d,
+                          int64_t pair_stride, const int32_t* row_index, float* out, cudaStream_t s) {
+    const size_t smem = sizeof(float) * (size_t)rows;
+    if (smem > 48 * 1024) return cudaErrorInvalidValue;
+    if (dtype == KS_DTYPE_BF16)
+        cosine_kernel<__nv_bfloat16><<<(unsigned)n_pairs, kCosThreads, smem, s>>>(
+            reinterpret_cast<const __nv_bfloat16*>(X), reinterpret_cast<const __nv_bfloat16*>(Y), rows, d,
+            pair_stride, row_index, out);
+    else
+        cosine_kernel<float><<<(unsigned)n_pairs, kCosThreads, smem, s>>>(
+            reinterpret_cast<const float*>(X), reinterpret_cast<const float*>(Y), rows, d, pair_stride,
+            row_index, out);
+    return cudaGetLastError();
+}
+
+// ----------------------------------------------------------------- knapsack
+constexpr int kMaxItems = 256;
+constexpr int kKnapThreads = 512;
+
+struct KnapArgs {
+    int kind;                 // 0 latency model, 1 explicit units
+    double c1, c2, c3;
+    long long n;              // context length
+    int n_items;
+    int budget;               // used when budget_frac < 0
+    double budget_frac;       // >= 0: budget = floor(frac * sum w)
+    int units[kMaxItems];
+    const float* sims;
+    uint8_t* mask;
+    double* objective;
+    int32_t* weights_out;
+    int32_t* budget_out;      // optional: the budget used
+    long long* best;          // scratch [2][cap + 1]
+    uint8_t* take;            // scratch [n_items][cap + 1]
+    int cap;                  // capacity of the scratch tables
+};
+
+__global__ void __launch_bounds__(kKnapThreads) knapsack_kernel(const KnapArgs a) {
+    __shared__ int w[kMaxItems];
+    __shared__ long long q[kMaxItems];
+    __shared__ int B;
+    const int tid = threadIdx.x;
+    const int N = a.n_items;
+    if (tid == 0) {
+        int wa = 1, wm = 1;
+        if (a.kind == 0) {
+            // Sec. 3.4: Delta = min(t_Attn(n), t_MLP), w = round(t / Delta), >= 1
+            // explicit _rn intrinsics: no FMA contraction, the same two
+            // roundings as c2 * n + c3 evaluated left to right
+            const double ta = __dadd_rn(__dmul_rn(a.c2, (double)a.n), a.c3);
+            const double tm = a.c1;
+            const double delta = fmin(ta, tm);
+            wa = (int)llround(__ddiv_rn(ta, delta));
+            wm = (int)llround(__ddiv_rn(tm, delta));
+            if (wa < 1) wa = 1;
+            if (wm < 1) wm = 1;
+        }
+        long long sum = 0;
+        for (int i = 0; i < N; ++i) {
+            // 0-based item i is sublayer i + 1: even i -> Attn, odd i -> MLP
+            w[i] = (a.kind == 0) ? ((i % 2 == 0) ? wa : wm) : a.units[i];
+            sum += w[i];
+        }
+        long long b = a.budget;
+        if (a.budget_frac >= 0.0) b = (long long)floor(__dmul_rn(a.budget_frac, (double)sum));
+        if (b > a.cap) b = a.cap;
+        if (b < 0) b = 0;
+        B = (int)b;
+        if (a.budget_out) *a.budget_out = (int)b;
+    }
+    for (int i = tid; i < N; i += blockDim.x) {
+        // q_i = round((1 - sigma_i) * 2^30), half away from zero, in double
+        const double v = __dmul_rn(__dsub_rn(1.0, (double)a.sims[i]), 1073741824.0);
+        q[i] = llround(v);
+    }
+    __syncthreads();
+    const int cap1 = B + 1;
+    long long* cur = a.best;
+    long long* nxt = a.best + (a.cap + 1);
+    for (int c = tid; c < cap1; c += blockDim.x) cur[c] = 0;
+    __syncthreads();
+    for (int i = 0; i < N; ++i) {
+        const int wi = w[i];
+        const long long qi = q[i];
+        uint8_t* tk = a.take + (size_t)i * (a.cap + 1);
+        for (int c = tid; c < cap1; c += blockDim.x) {
+            long long v = cur[c];
+            uint8_t t = 0;
+            if (c >= wi) {
+                const long long cand = cur[c - wi] + qi;
+                if (cand > v) {
+                    v = cand;
+                    t = 1;
+                }
+            }
+            nxt[c] = v;
+            tk[c] = t;
+        }
+        __syncthreads();
+        long long* tmp = cur;
+        cur = nxt;
+        nxt = tmp;
+    }
+    if (tid == 0) {
+        int c = B;
+        for (int i = N - 1; i >= 0; --i) {
+            const uint8_t t = a.take[(size_t)i * (a.cap + 1) + c];
+            a.mask[i] = t;
+            if (t) c -= w[i];
+        }
+        if (a.objective) *a.objective = (double)cur[B] / 1073741824.0;
+    }
+    if (a.weights_out)
+        for (int i = tid; i < N; i += blockDim.x) a.weights_out[i] = w[i];
+}
+
+size_t select_scratch_bytes(int n_items, int cap) {
+    const size_t best = sizeof(long long) * 2 * ((size_t)cap + 1);
+    const size_t take = (size_t)n_items * ((size_t)cap + 1);
+    return ((best + take + 255) / 256) * 256;
+}
+
+cudaError_t launch_select(const ks_latency* lat, const float* sims, int64_t n, int n_items, int budget,
+                          double budget_frac, uint8_t* mask, double* objective, int32_t* weights,
+                          int32_t* budget_out, void* scratch, int cap, cudaStream_t s) {
+    KnapArgs a{};
+    a.kind = lat->kind;
+    a.c1 = lat->c1;
+    a.c2 = lat->c2;
+    a.c3 = lat->c3;
+    a.n = n;
+    a.n_items = n_items;
+    a.budget = budget;
+    a.budget_frac = budget_frac;
+    if (lat->kind == 1)
+        for (int i = 0; i < n_items; ++i) a.units[i] = lat->units[i];
+    a.sims = sims;
+    a.mask = mask;
+    a.objective = objective;
+    a.weights_out = weights;
+    a.budget_out = budget_out;
+    a.cap = cap;
+    a.best = reinterpret_cast<long long*>(scratch);
+    a.take = reinterpret_cast<uint8_t*>(scratch) + sizeof(long long) * 2 * ((size_t)cap + 1);
+    knapsack_kernel<<<1, kKnapThreads, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace ks
+
+// ------------------------------------------------------------------- C ABI
+using namespace ks;
+
+extern "C" ks_status ks_cosine(const void* X, const void* Y, int32_t dtype, int64_t n_pairs, int32_t rows,
+                               int32_t d, int64_t pair_stride, const int32_t* row_index, float* out,
+                               void* stream) {
+    if (!X || !Y || !out) {
+        set_error("ks_cosine: null pointer");
+        return KS_ERR_INVALID_ARG;
+    }
+    if (n_pairs < 1 || n_pairs > (1 << 30) || rows < 1 || rows > 8192 || d < 1 || pair_stride < 0 ||
+        (dtype != KS_DTYPE_F32 && dtype != KS_DTYPE_BF16)) {
+        set_error("ks_cosine: bad size or dtype");
+        return KS_ERR_INVALID_ARG;
+    }
+    cudaError_t e = launch_cosine(X, Y, dtype, n_pairs, rows, d, pair_stride, row_index, out,
+                                  reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) {
+        set_error("ks_cosine: %s", cudaGetErrorString(e));
+        return KS_ERR_CUDA;
+    }
+    return KS_OK;
+}
+
+extern "C" size_t ks_select_scratch_bytes(int32_t n_sublayers, int32_t budget_units) {
+    if (n_sublayers < 2 || n_sublayers > kMaxItems || budget_units < 0 || budget_units > 65535) return 0;
+    return select_scratch_bytes(n_sublayers, budget_units);
+}
+
+static ks_status check_latency(const ks_latency* lat, int32_t n) {
+    if (!lat) return KS_ERR_INVALID_ARG;
+    if (lat->kind == 0) {
+        if (!(lat->c1 > 0.0) || !(lat->c2 >= 0.0) || !(lat->c3 >= 0.0) || !std::isfinite(lat->c1) ||
+            !std::isfinite(lat->c2) || !std::isfinite(lat->c3))
+            return KS_ERR_INVALID_ARG;
+        return KS_OK;
+    }
+    if (lat->kind == 1) {
+        if (!lat->units) return KS_ERR_INVALID_ARG;
+        for (int i = 0; i < n; ++i)
+            if (lat->units[i] < 1 || lat->units[i] > 65535) return KS_ERR_INVALID_ARG;
+        return KS_OK;
+    }
+    return KS_ERR_INVALID_ARG;
+}
+
+extern "C" ks_status ks_select_mask(const ks_latency* lat, const float* sims, int64_t context_len,
+                                    int32_t n_sublayers, int32_t budget_units, uint8_t* mask_out,
+                                    double* objective_out, int32_t* weights_out, void* scratch,
+                                    size_t scratch_bytes, void* stream) {
+    if (!sims || !mask_out || !scratch) {
+        set_error("ks_select_mask: null pointer");
+        return KS_ERR_INVALID_ARG;
+    }
+    if (n_sublayers < 2 || n_sublayers > kMaxItems || (n_sublayers & 1) || budget_units < 0 ||
+        budget_units > 65535 || context_len < 0) {
+        set_error("ks_select_mask: bad n_sublayers / budget / context_len");
+        return KS_ERR_INVALID_ARG;
+    }
+    if (check_latency(lat, n_sublayers) != KS_OK) {
+        set_error("ks_select_mask: bad latency model");
+        return KS_ERR_INVALID_ARG;
+    }
+    if ((reinterpret_cast<uintptr_t>(scratch) & 15) != 0) {
+        set_error("ks_select_mask: scratch must be 16-byte aligned");
+        return KS_ERR_INVALID_ARG;
+    }
+    if (scratch_bytes < select_scratch_bytes(n_sublayers, budget_units)) {
+        set_error("ks_select_mask: scratch too small");
+        return KS_ERR_WORKSPACE;
+    }
+    cudaError_t e = launch_select(lat, sims, context_len, n_sublayers, budget_units, -1.0, mask_out,
+                                  objective_out, weights_out, nullptr, scratch, budget_units,
+                                  reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) {
+        set_error("ks_select_mask: %s", cudaGetErrorString(e));
+        return KS_ERR_CUDA;
+    }
+    return KS_OK;
+}

@@ -1,0 +1,241 @@
+"""GPU parity of a1-a3 (draft, verify, acceptance) and the history states
+against the oracle, plus the lossless invariant on the GPU itself.
+
+* Tiny fp32 workload (4 layers, 256-token prompt, 32 tokens, gamma 4): logits
+  within 1e-4 relative, tokens equal to the oracle's wherever the oracle's
+  top-2 margin exceeds 1e-3.
+* Small bf16 models (ragged d_ff, 300-token prompts spanning three attention
+  chunks, QK-norm on and off, head_dim 64 and 128): logits within 2e-2
+  relative (the workload tolerance), tokens under the same margin rule.
+* Lossless (Sec. 2.1): speculative output is bit-identical to the GPU's own
+  greedy decode for every mask and the knapsack policy; a full-mask draft
+  reproduces the target's logits bit for bit."""
+import numpy as np
+import pytest
+
+from helpers import need_gpu, oracle_model, rel_err, token_ok
+from oracle import decoder as D
+from oracle import select as S
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _gpu():
+    need_gpu()
+
+
+def small_bf16(hd=128, qk_norm=False, L=2):
+    from paper_2602_20217_gb300.configs import ModelShape
+    return ModelShape(f"small-bf16-hd{hd}", L, 512, 8, 2, hd, 1368, 2048, qk_norm=qk_norm,
+                      dtype="bf16", rope_theta=500000.0)
+
+
+def make(shape, max_seq, seed=0):
+    from paper_2602_20217_gb300.model import Model
+    return Model(shape, max_seq=max_seq, seed=seed)
+
+
+# --------------------------------------------------------------- tiny fp32
+@pytest.fixture(scope="module")
+def tiny():
+    from paper_2602_20217_gb300 import synth
+    from paper_2602_20217_gb300.configs import TINY
+    prompt = synth.prompt_tokens(TINY, 256, seed=1)
+    cfg, w = oracle_model(TINY, seed=0)
+    return TINY, prompt, cfg, w
+
+
+def test_tiny_prefill_kv_and_pending(tiny):
+    shape, prompt, cfg, w = tiny
+    m = make(shape, 512)
+    pend = m.prefill(prompt)
+    s = D.Session(cfg, w, 512)
+    logits, _ = s.forward(prompt, 0)
+    assert token_ok(pend, logits[-1], 1e-3)
+    assert rel_err(m.logits(16), logits[-16:]) < 1e-4
+    for layer in (0, 3):
+        for which, ref in (("k", s.k[layer]), ("v", s.v[layer])):
+            got = m.kv(layer, 0, 256, which)
+            assert np.max(np.abs(got - ref[:, :256])) <= 1e-4 * np.max(np.abs(ref[:, :256]))
+    m.close()
+
+
+def test_tiny_greedy_matches_oracle(tiny):
+    shape, prompt, cfg, w = tiny
+    m = make(shape, 512)
+    m.prefill(prompt)
+    toks = m.decode_greedy(32)
+    s = D.Session(cfg, w, 512)
+    ref = [s.prefill(prompt)]
+    for i in range(31):
+        logits, _ = s.forward([ref[-1]], s.p)
+        s.p += 1
+        assert token_ok(toks[i + 1], logits[0], 1e-3), i
+        ref.append(int(toks[i + 1]))     # follow the GPU's token (equal unless a near-tie)
+    assert list(toks) == ref
+    m.close()
+
+
+@pytest.mark.parametrize("mask_kind", ["attn_skip", "random", "full"])
+def test_tiny_draft_and_verify_match_oracle(tiny, mask_kind):
+    shape, prompt, cfg, w = tiny
+    n = shape.n_sublayers
+    mask = {"attn_skip": np.array([0, 1] * shape.n_layers, np.uint8),
+            "random": np.array([1, 1, 0, 1, 1, 0, 0, 1], np.uint8),
+            "full": np.ones(n, np.uint8)}[mask_kind]
+    m = make(shape, 512)
+    m.prefill(prompt)
+    s = D.Session(cfg, w, 512)
+    s.prefill(prompt)
+    for step in range(4):
+        drafts = m.draft(mask, 4)
+        # the oracle drafts from the same state
+        ref_drafts = []
+        tok = s.pending
+        for t in range(4):
+            lg, _ = s.forward([tok], s.p + t, mask=mask)
+            assert token_ok(drafts[t], lg[0], 1e-3)
+            tok = int(drafts[t])
+            ref_drafts.append(tok)
+        a, new = m.verify(None, 4)
+        vlog = m.logits(5)
+        ra, rnew = s.verify(ref_drafts)
+        rl, _ = s.forward([s.pending], s.p)  # noqa: F841  (keeps the session moving)
+        assert (a, list(new)) == (ra, list(rnew)), step
+        if mask_kind == "full":
+            assert a == 4
+        assert vlog.shape == (5, shape.vocab)
+    m.close()
+
+
+def test_tiny_verify_logits_and_history(tiny):
+    shape, prompt, cfg, w = tiny
+    m = make(shape, 512)
+    m.prefill(prompt)
+    s = D.Session(cfg, w, 512)
+    s.prefill(prompt)
+    # teacher-forced verify with the oracle's own greedy continuation
+    for step in range(6):
+        lg = []
+        tok = s.pending
+        toks = []
+        probe = D.Session(cfg, w, 512)
+        probe.k = [k.copy() for k in s.k]
+        probe.v = [v.copy() for v in s.v]
+        probe.p, probe.pending = s.p, s.pending
+        for t in range(3):
+            probe.ar_step()
+            toks.append(probe.pending)
+        drafts = toks if step % 2 == 0 else [toks[0], (toks[1] + 1) % shape.vocab, toks[2]]
+        a, new = m.verify(drafts, 3)
+        got = m.logits(4)
+        ref_logits, _ = s.forward([s.pending] + drafts, s.p)
+        assert rel_err(got, ref_logits) < 1e-4
+        ra, rnew = s.verify(drafts)
+        assert (a, list(new)) == (ra, list(rnew))
+    hist = m.history()
+    ref = s.history()
+    assert hist.shape == ref.shape
+    assert np.max(np.abs(hist - ref)) <= 1e-4 * np.max(np.abs(ref))
+    sims, r = m.history_similarities()
+    assert r == ref.shape[1]
+    assert np.max(np.abs(sims - S.sublayer_similarities(ref))) < 1e-3
+    m.close()
+
+
+def test_tiny_lossless_and_knapsack_policy(tiny):
+    from paper_2602_20217_gb300 import knapspec as ks
+    from paper_2602_20217_gb300 import synth
+    shape, prompt, cfg, w = tiny
+    m = make(shape, 512)
+    m.prefill(prompt)
+    ar = m.decode_greedy(32)
+    rng = np.random.default_rng(0)
+    masks = [np.zeros(8, np.uint8), np.ones(8, np.uint8), np.array([0, 1] * 4, np.uint8),
+             rng.integers(0, 2, 8).astype(np.uint8)]
+    for mask in masks:
+        for gamma in (1, 4, 7):
+            m.prefill(prompt)
+            out, st, acc = m.generate(32, gamma, mask=mask)
+            assert list(out) == list(ar), (mask, gamma)
+            assert st.steps == len(acc) and st.accepted == int(acc.sum())
+            if mask.all():
+                assert all(a == gamma for a in acc[:-1])
+    # knapsack policy with the workload's seeded units and budget 5
+    units = synth.unit_table(8, seed=2)
+    lat = ks.latency(1, units=units)
+    for T in (1, 3):
+        m.prefill(prompt)
+        out, st, acc = m.generate(32, 4, latency=lat, budget_frac=5 / units.sum(), resolve_every=T)
+        assert list(out) == list(ar)
+        assert st.resolves == (st.steps + T - 1) // T
+    m.close()
+
+
+# ------------------------------------------------------------- small bf16
+@pytest.mark.parametrize("hd,qk_norm", [(128, False), (128, True), (64, True)])
+def test_bf16_logits_tokens_and_lossless(hd, qk_norm):
+    from paper_2602_20217_gb300 import synth
+    shape = small_bf16(hd, qk_norm)
+    prompt = synth.prompt_tokens(shape, 300, seed=1)
+    cfg, w = oracle_model(shape, seed=0)
+    m = make(shape, 512)
+    pend = m.prefill(prompt)
+    s = D.Session(cfg, w, 512)
+    logits, _ = s.forward(prompt, 0)
+    assert rel_err(m.logits(16), logits[-16:]) < 2e-2
+    assert token_ok(pend, logits[-1], 0.05 * np.max(np.abs(logits[-1])))
+    s.p, s.pending = 300, pend
+    # teacher-forced verify rows vs oracle (R = 5), then AR == spec on the GPU
+    drafts = list(synth.prompt_tokens(shape, 4, seed=9))
+    m.verify(drafts, 4)
+    ref, _ = s.forward([pend] + drafts, 300)
+    assert rel_err(m.logits(5), ref) < 2e-2
+    # lossless on the GPU
+    m.prefill(prompt)
+    ar = m.decode_greedy(40)
+    for mask in (np.array([0, 1] * shape.n_layers, np.uint8), np.array([1, 0, 0, 1], np.uint8)):
+        m.prefill(prompt)
+        out, st, acc = m.generate(40, 5, mask=mask)
+        assert list(out) == list(ar)
+    m.close()
+
+
+def test_bf16_full_mask_draft_equals_target_bitwise():
+    from paper_2602_20217_gb300 import synth
+    shape = small_bf16(128, True)
+    prompt = synth.prompt_tokens(shape, 260, seed=3)
+    m = make(shape, 512)
+    m.prefill(prompt)
+    full = np.ones(shape.n_sublayers, np.uint8)
+    d = m.draft(full, 1)
+    draft_logits = m.logits(1).copy()
+    a, new = m.verify(None, 1)
+    verify_logits = m.logits(2)
+    assert np.array_equal(draft_logits[0], verify_logits[0])
+    assert a == 1 and new[0] == d[0]
+    m.close()
+
+
+def test_capacity_and_state_errors():
+    from paper_2602_20217_gb300 import knapspec as ks
+    from paper_2602_20217_gb300.configs import TINY
+    m = make(TINY, 64)
+    with pytest.raises(ks.KsError) as e:
+        m.draft(np.ones(8, np.uint8), 4)
+    assert e.value.status == ks.KS_ERR_STATE
+    with pytest.raises(ks.KsError) as e:
+        m.prefill(np.zeros(64, np.int32))
+    assert e.value.status == ks.KS_ERR_CAPACITY
+    m.prefill(np.arange(60, dtype=np.int32))
+    with pytest.raises(ks.KsError) as e:
+        m.draft(np.ones(8, np.uint8), 4)
+    assert e.value.status == ks.KS_ERR_CAPACITY
+    with pytest.raises(ks.KsError) as e:
+        m.verify(None, 2)
+    assert e.value.status == ks.KS_ERR_STATE
+    with pytest.raises(ks.KsError) as e:
+        m.prefill(np.array([5, 2000], np.int32))
+    assert e.value.status == ks.KS_ERR_INVALID_ARG
+    m.close()
