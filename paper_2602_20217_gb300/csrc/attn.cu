@@ -15,14 +15,15 @@
 // staged in shared memory with cp.async (zero-filled past the valid keys).
 // bf16 models: S = Q K^T and O += P V on mma.sync.m16n8k16 with fp32 online
 // softmax in the log2 domain.  fp32 models: CUDA-core dot products.
-// Partials (m, l, o) per (row, query head, chunk) are merged in chunk order
-// by attn_merge_kernel.
+// Partials (m, l, o) per (row, query head, chunk) are merged by
+// attn_merge_kernel in a fixed order.
 #include "common.cuh"
 #include "internal.h"
 
 namespace ks {
 
 constexpr int kAttnWarps = 4;
+constexpr int kPartPad = 4;  // partial row: m, l, 2 pad, o[hd] (16-byte aligned o)
 constexpr float kLog2e = 1.4426950408889634f;
 
 // ------------------------------------------------------------ small helpers
@@ -125,7 +126,7 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const AttnArgs a) {
     __nv_bfloat16* Qs = reinterpret_cast<__nv_bfloat16*>(smem);
     __nv_bfloat16* Ks = Qs + (size_t)mpad * P;
     __nv_bfloat16* Vs = Ks + (size_t)C * P;
-    float* wpart = reinterpret_cast<float*>(Vs + (size_t)C * P);  // [4][16][HD + 2]
+    float* wpart = reinterpret_cast<float*>(Vs + (size_t)C * P);  // [4][16][HD + 2] (m, l, o)
 
     // 1. new K/V rows of this chunk -> cache (generic stores, then barrier)
     write_new_kv<__nv_bfloat16, NPL>(a, h, cs, ce);
@@ -305,8 +306,8 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const AttnArgs a) {
                 }
             }
             const int r = m / G, gq = m - r * G;
-            float* dst = a.part + (((size_t)r * a.hq + h * G + gq) * a.n_chunks_max + c) * (HD + 2);
-            dst[col] = out;
+            float* dst = a.part + (((size_t)r * a.hq + h * G + gq) * a.n_chunks_max + c) * (HD + kPartPad);
+            dst[col < 2 ? col : col + 2] = out;
         }
         __syncthreads();
     }
@@ -365,11 +366,11 @@ __global__ void __launch_bounds__(128) attn_f32_kernel(const AttnArgs a) {
         }
         l = warp_sum(l);
         __syncwarp();
-        float* dst = a.part + (((size_t)r * a.hq + h * G + gq) * a.n_chunks_max + c) * (HD + 2);
+        float* dst = a.part + (((size_t)r * a.hq + h * G + gq) * a.n_chunks_max + c) * (HD + kPartPad);
         for (int d = lane; d < HD; d += 32) {
             float acc = 0.f;
             for (int j = 0; j < kend - cs; ++j) acc = fmaf(psh[warp][j], vc[(size_t)(cs + j) * HD + d], acc);
-            dst[2 + d] = acc;
+            dst[kPartPad + d] = acc;
         }
         if (lane == 0) {
             dst[0] = mx;
@@ -381,26 +382,62 @@ __global__ void __launch_bounds__(128) attn_f32_kernel(const AttnArgs a) {
 
 // ------------------------------------------------------------------ merge
 // out[r][hq_idx * hd + d] = sum_c 2^(m_c - M) o_c[d] / sum_c 2^(m_c - M) l_c over
-// the chunks 0 .. pos_r / C of row r, in chunk order.
+// the chunks 0 .. pos_r / C of row r.  Fixed order for every term: the max is
+// exact in any order; l and o are summed per thread (stride 128 over chunks)
+// or per warp (chunks c = w mod 4) and then in thread / warp order.  The
+// chunk count depends only on the row's position, so a row gives the same
+// bits in a 1-row pass and in a gamma+1-row pass.
 template <typename WT, int HD>
-__global__ void __launch_bounds__(HD) attn_merge_kernel(const AttnArgs a) {
-    const int hq_idx = blockIdx.x, r = blockIdx.y, d = threadIdx.x;
+__global__ void __launch_bounds__(128) attn_merge_kernel(const AttnArgs a) {
+    extern __shared__ float wsh[];           // [nch] chunk weights
+    __shared__ float red[kAttnWarps + 1];
+    __shared__ float osh[kAttnWarps][HD];
+    const int hq_idx = blockIdx.x, r = blockIdx.y;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int pos = a.p0 + r;
     const int nch = pos / kAttnChunk + 1;
-    const float* base = a.part + ((size_t)r * a.hq + hq_idx) * a.n_chunks_max * (HD + 2);
+    constexpr int S = HD + kPartPad;
+    const float* base = a.part + ((size_t)r * a.hq + hq_idx) * a.n_chunks_max * S;
     float mx = -INFINITY;
-    for (int c = 0; c < nch; ++c) mx = fmaxf(mx, base[(size_t)c * (HD + 2)]);
-    float L = 0.f, O = 0.f;
-    for (int c = 0; c < nch; ++c) {
-        const float* p = base + (size_t)c * (HD + 2);
-        const float m = p[0];
-        if (m == -INFINITY) continue;
-        const float w = exp2f(m - mx);
-        L += w * p[1];
-        O += w * p[2 + d];
+    for (int c = tid; c < nch; c += blockDim.x) mx = fmaxf(mx, base[(size_t)c * S]);
+    mx = warp_max(mx);
+    if (lane == 0) red[warp] = mx;
+    __syncthreads();
+    mx = fmaxf(fmaxf(red[0], red[1]), fmaxf(red[2], red[3]));
+    float ls = 0.f;
+    for (int c = tid; c < nch; c += blockDim.x) {
+        const float m = base[(size_t)c * S];
+        const float w = (m == -INFINITY) ? 0.f : exp2f(m - mx);
+        wsh[c] = w;
+        ls = fmaf(w, base[(size_t)c * S + 1], ls);
     }
+    const float L = block_sum<kAttnWarps>(ls, red);   // ends with a barrier: wsh is visible
+    constexpr int PER = HD / 32;                      // dims per lane
+    float o[PER];
+#pragma unroll
+    for (int i = 0; i < PER; ++i) o[i] = 0.f;
+    for (int c = warp; c < nch; c += kAttnWarps) {
+        const float w = wsh[c];
+        const float* src = base + (size_t)c * S + kPartPad + PER * lane;
+        if constexpr (PER == 4) {
+            const float4 v = *reinterpret_cast<const float4*>(src);
+            o[0] = fmaf(w, v.x, o[0]);
+            o[1] = fmaf(w, v.y, o[1]);
+            o[2] = fmaf(w, v.z, o[2]);
+            o[3] = fmaf(w, v.w, o[3]);
+        } else {
+#pragma unroll
+            for (int i = 0; i < PER; ++i) o[i] = fmaf(w, src[i], o[i]);
+        }
+    }
+#pragma unroll
+    for (int i = 0; i < PER; ++i) osh[warp][PER * lane + i] = o[i];
+    __syncthreads();
     WT* out = reinterpret_cast<WT*>(a.out);
-    out[(size_t)r * a.out_ld + hq_idx * HD + d] = from_float<WT>(O / L);
+    for (int d = tid; d < HD; d += blockDim.x) {
+        const float O = ((osh[0][d] + osh[1][d]) + osh[2][d]) + osh[3][d];
+        out[(size_t)r * a.out_ld + hq_idx * HD + d] = from_float<WT>(O / L);
+    }
 }
 
 // --------------------------------------------------------------- launchers
@@ -436,12 +473,15 @@ cudaError_t launch_attention(int dtype, const AttnArgs& a, cudaStream_t s) {
 
 cudaError_t launch_attn_merge(int dtype, const AttnArgs& a, cudaStream_t s) {
     dim3 grid(a.hq, a.R);
+    const int nch = (a.p0 + a.R - 1) / kAttnChunk + 1;
+    const size_t smem = sizeof(float) * (size_t)nch;
+    if (smem > 48 * 1024) return cudaErrorInvalidValue;
     if (dtype == 1) {
-        if (a.hd == 128) attn_merge_kernel<__nv_bfloat16, 128><<<grid, 128, 0, s>>>(a);
-        else attn_merge_kernel<__nv_bfloat16, 64><<<grid, 64, 0, s>>>(a);
+        if (a.hd == 128) attn_merge_kernel<__nv_bfloat16, 128><<<grid, 128, smem, s>>>(a);
+        else attn_merge_kernel<__nv_bfloat16, 64><<<grid, 128, smem, s>>>(a);
     } else {
-        if (a.hd == 128) attn_merge_kernel<float, 128><<<grid, 128, 0, s>>>(a);
-        else attn_merge_kernel<float, 64><<<grid, 64, 0, s>>>(a);
+        if (a.hd == 128) attn_merge_kernel<float, 128><<<grid, 128, smem, s>>>(a);
+        else attn_merge_kernel<float, 64><<<grid, 128, smem, s>>>(a);
     }
     return cudaGetLastError();
 }

@@ -1,6 +1,8 @@
 // Internal interfaces between the translation units of libknapspec.
 #pragma once
 
+#include <cuda.h>
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -12,31 +14,45 @@ namespace ks {
 enum GemvEpi { EPI_STORE = 0, EPI_RESID = 1, EPI_SWIGLU = 2, EPI_LMHEAD = 3 };
 
 struct GemvArgs {
+    CUtensorMap wmap;       // bf16: TMA map of W (dims {K, rows}, box 256 x 16)
+    CUtensorMap xmap;       // bf16: TMA map of the input rows (dims {K, max_rows}, box 256 x 8 or 16)
+    int dtype;              // KS_DTYPE_F32 / KS_DTYPE_BF16 (selects kernel and split plan)
     const void* W;          // [N (or 2N for SwiGLU)][K], row stride K, model dtype
     int N;                  // output features (SwiGLU: d_ff; rows n and N + n pair up)
     int K;
     int R;                  // activation rows, 1..16
     int ksplit;             // K slices (grid.y); set by gemv_plan
     int kc;                 // K per slice (multiple of 64)
-    const void* in;         // fp32 residual [R][in_ld] when norm_gain != null, else model dtype [R][in_ld]
+    const void* in;         // fp32: the residual [R][in_ld] when norm_gain != null, else the input;
+                            // bf16: the input in bf16 [R][in_ld] (x * gain when ss_in != null)
     int in_ld;
     const void* norm_gain;  // RMSNorm gain [K] (model dtype) or null
     float eps;
+    const float* ss_in;     // with norm_gain: per-64-feature sums of squares [ss_groups][16]
+    int ss_groups;
+    float* ss_out;          // EPI_RESID: sums of squares of the new residual [groups][16]
+    __nv_bfloat16* xg_out;  // EPI_RESID (bf16): new residual times next_gain, the next GEMV's input
+    const void* next_gain;  // gain of the next RMSNorm (model dtype)
+    int* err;               // device status word: set to 1 when a bounded wait gives up
     float* out; int out_ld;                    // EPI_STORE (fp32)
     float* resid; int resid_ld;                // EPI_RESID: resid[r][n] += y
     float* capture; long long capture_ld;      // EPI_RESID: optional copy of the new residual
     void* act; int act_ld;                     // EPI_SWIGLU: silu(gate) * up, model dtype
     float* logits; int logits_ld;              // EPI_LMHEAD
-    float* amax_val; int* amax_idx;            // EPI_LMHEAD per-CTA partials [grid.x][16]
+    float* amax_val; int* amax_idx;            // EPI_LMHEAD per-group candidates [groups][16]
     int* tokens;                               // EPI_LMHEAD argmax per row
     float* partial;                            // split-K partials [ksplit][R][N or 2N]
-    int* counters;                             // per-CTA-column arrival counters (+1 global)
+    int* counters;                             // [0] work queue, [1] finished CTAs, [2 + g] group tickets
 };
 
-void gemv_plan(GemvArgs& a, int epi);           // choose ksplit / kc from (N, K) only
-size_t gemv_partial_floats(int N, int K, int R, int epi);
+void gemv_plan(GemvArgs& a, int epi);           // choose ksplit / kc from (N, K, dtype) only
+size_t gemv_partial_floats(int N, int K, int R, int epi, int dtype);
 int gemv_grid_x(int N);
 cudaError_t launch_gemv(int dtype, int epi, const GemvArgs& a, cudaStream_t s);
+// TMA map of a row-major bf16 matrix [rows][K] (K % 8 == 0, 16-byte aligned
+// base), box 256 columns x box_rows rows, no swizzle, zero fill outside.
+bool make_tma_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t K, uint32_t box_rows);
+int gemv_groups(int N, int dtype);              // output groups (argmax candidates) of a launch
 
 // ------------------------------------------------------------- attention
 struct AttnArgs {
@@ -53,7 +69,7 @@ struct AttnArgs {
     const void* k_norm;
     float eps;
     int chunk;              // keys per CTA (fixed; split boundaries are absolute)
-    float* part;            // [R][hq][n_chunks_max][hd + 2] (m, l, o[hd])
+    float* part;            // [R][hq][n_chunks_max][hd + 4] (m, l, pad, pad, o[hd])
     int n_chunks_max;
     void* out;              // [R][hq hd] model dtype: merged attention output
     int out_ld;
@@ -62,6 +78,7 @@ struct AttnArgs {
 cudaError_t launch_attention(int dtype, const AttnArgs& a, cudaStream_t s);
 cudaError_t launch_attn_merge(int dtype, const AttnArgs& a, cudaStream_t s);
 constexpr int kAttnChunk = 128;
+constexpr int kSsGroup = 16;    // features per sum-of-squares partial (= rows of a bf16 GEMV work item)
 
 // ---------------------------------------------------------------- select
 cudaError_t launch_cosine(const void* X, const void* Y, int dtype, int64_t n_pairs, int rows,

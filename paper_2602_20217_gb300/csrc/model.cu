@@ -40,9 +40,12 @@ enum { K_QKV = 0, K_ATTN, K_MERGE, K_OPROJ, K_GATEUP, K_DOWN, K_LMHEAD, K_EMBED,
 
 // ------------------------------------------------------------ small kernels
 // x[r] = embed[tok[r]] (fp32); optionally copied to the history plane 0.
+// Also the per-64-feature sums of squares ss[g][r] that the next RMSNorm
+// uses (lane l adds features 64 g + l and 64 g + 32 + l, then a butterfly -
+// the same order as the residual epilogues).
 template <typename WT>
 __global__ void embed_kernel(const WT* embed, const int32_t* tok, int d, int vocab, float* x,
-                             float* capture) {
+                             float* capture, float* ss, __nv_bfloat16* xg, const WT* next_gain) {
     const int r = blockIdx.x;
     int t = tok[r];
     if (t < 0 || t >= vocab) t = 0;
@@ -51,6 +54,22 @@ __global__ void embed_kernel(const WT* embed, const int32_t* tok, int d, int voc
         const float v = to_float(e[k]);
         x[(size_t)r * d + k] = v;
         if (capture) capture[(size_t)r * d + k] = v;
+        if (xg) xg[(size_t)r * d + k] = __float2bfloat16_rn(v * to_float(next_gain[k]));
+    }
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int groups = (d + kSsGroup - 1) / kSsGroup;
+    // two 16-feature groups per warp pass: lanes 0-15 and 16-31
+    for (int gp = 2 * warp; gp < groups; gp += 2 * (blockDim.x / 32)) {
+        const int q = gp + (lane >> 4);
+        const int n = q * kSsGroup + (lane & 15);
+        float s = 0.f;
+        if (q < groups && n < d) {
+            const float v = to_float(e[n]);
+            s = v * v;
+        }
+#pragma unroll
+        for (int o = 8; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+        if ((lane & 15) == 0 && q < groups) ss[q * 16 + r] = s;
     }
 }
 
@@ -73,7 +92,7 @@ __global__ void accept_kernel(int32_t* rows, const int32_t* z, int gamma, int32_
 static size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
 struct Layout {
-    size_t kv, rope, x, qkv, attn_out, act, attn_part, gemv_part, counters, logits, amax_val,
+    size_t kv, rope, x, ss, xg, qkv, attn_out, act, attn_part, gemv_part, counters, logits, amax_val,
         amax_idx, tok, hist, hist_idx, sims, mask, obj, wts, select, total;
     int n_chunks_max;
     size_t gemv_part_floats;
@@ -107,16 +126,17 @@ static Layout make_layout(const ks_config* c) {
     L.n_chunks_max = (c->max_seq + kAttnChunk - 1) / kAttnChunk;
     L.hist_slots = c->hist_steps + 1;
     size_t gp = 0;
-    gp = std::max(gp, gemv_partial_floats(nqkv, d, R, EPI_STORE));
-    gp = std::max(gp, gemv_partial_floats(d, c->n_q_heads * hd, R, EPI_RESID));
-    gp = std::max(gp, gemv_partial_floats(c->d_ff, d, R, EPI_SWIGLU));
-    gp = std::max(gp, gemv_partial_floats(d, c->d_ff, R, EPI_RESID));
+    gp = std::max(gp, gemv_partial_floats(nqkv, d, R, EPI_STORE, c->dtype));
+    gp = std::max(gp, gemv_partial_floats(d, c->n_q_heads * hd, R, EPI_RESID, c->dtype));
+    gp = std::max(gp, gemv_partial_floats(c->d_ff, d, R, EPI_SWIGLU, c->dtype));
+    gp = std::max(gp, gemv_partial_floats(d, c->d_ff, R, EPI_RESID, c->dtype));
+    gp = std::max(gp, gemv_partial_floats(c->vocab, d, R, EPI_LMHEAD, c->dtype));
     L.gemv_part_floats = gp;
     int gx = gemv_grid_x(c->vocab);
     gx = std::max(gx, gemv_grid_x(nqkv));
     gx = std::max(gx, gemv_grid_x(c->d_ff));
     gx = std::max(gx, gemv_grid_x(d));
-    L.counters_n = gx + 1;
+    L.counters_n = gx + 2;
 
     size_t off = 0;
     auto take = [&](size_t bytes) {
@@ -127,16 +147,18 @@ static Layout make_layout(const ks_config* c) {
     L.kv = take(2 * (size_t)c->n_layers * c->n_kv_heads * (size_t)c->max_seq * hd * es);
     L.rope = take(sizeof(float) * (size_t)c->max_seq * hd);
     L.x = take(sizeof(float) * (size_t)R * d);
+    L.ss = take(sizeof(float) * 16 * (size_t)((d + kSsGroup - 1) / kSsGroup));
+    L.xg = take(sizeof(__nv_bfloat16) * (size_t)R * d);
     L.qkv = take(sizeof(float) * (size_t)R * nqkv);
     L.attn_out = take(es * (size_t)R * c->n_q_heads * hd);
     L.act = take(es * (size_t)R * c->d_ff);
-    L.attn_part = take(sizeof(float) * (size_t)R * c->n_q_heads * L.n_chunks_max * (hd + 2));
+    L.attn_part = take(sizeof(float) * (size_t)R * c->n_q_heads * L.n_chunks_max * (hd + 4));
     L.gemv_part = take(sizeof(float) * std::max<size_t>(gp, 1));
     L.counters = take(sizeof(int) * (size_t)L.counters_n);
     L.logits = take(sizeof(float) * (size_t)R * c->vocab);
-    L.amax_val = take(sizeof(float) * (size_t)gemv_grid_x(c->vocab) * 16);
-    L.amax_idx = take(sizeof(int) * (size_t)gemv_grid_x(c->vocab) * 16);
-    // tokens: rows[R+1] | target[R] | result[R+3] | prompt/out[max_seq]
+    L.amax_val = take(sizeof(float) * (size_t)gemv_groups(c->vocab, c->dtype) * 16);
+    L.amax_idx = take(sizeof(int) * (size_t)gemv_groups(c->vocab, c->dtype) * 16);
+    // tokens: rows[R+1] | target[R] | result[R+3] | err | prompt/out[max_seq]
     L.tok = take(sizeof(int) * ((size_t)3 * R + 8 + c->max_seq));
     L.hist = take(sizeof(float) * (size_t)(nsub + 1) * L.hist_slots * R * d);
     L.hist_idx = take(sizeof(int) * (size_t)L.hist_slots * R);
@@ -174,9 +196,10 @@ struct ks_model {
     Layout lay;
     // carved pointers
     char* kv;
-    float *rope, *x, *qkv, *attn_part, *gemv_part, *logits, *amax_val, *hist, *sims;
+    float *rope, *x, *ss, *qkv, *attn_part, *gemv_part, *logits, *amax_val, *hist, *sims;
+    __nv_bfloat16* xg;
     void *attn_out, *act, *select;
-    int *counters, *amax_idx, *rows, *target, *result, *seq, *hist_idx;
+    int *counters, *amax_idx, *rows, *target, *result, *err, *seq, *hist_idx;
     uint8_t* mask_dev;
     double* obj_dev;
     int* wts_dev;
@@ -193,6 +216,9 @@ struct ks_model {
     int hist_next = 0;
     int64_t launches = 0;
     int64_t h2d = 0, d2h = 0;
+    // bf16: TMA maps of every weight matrix and of the three projection inputs
+    std::vector<CUtensorMap> map_qkv, map_o, map_gu, map_down;
+    CUtensorMap map_lm, map_xg[2], map_attn_out[2], map_act[2];  // [0]: 8-row boxes, [1]: 16-row boxes
     KlassTiming timing[kKlasses];
 };
 
@@ -263,30 +289,81 @@ static ks_status forward(ks_model* m, const int32_t* tok, int R, int p0, const u
     const int d = c.d_model, hd = c.head_dim;
     const int nqkv = (c.n_q_heads + 2 * c.n_kv_heads) * hd;
     const int dt = m->dtype;
+    const bool bf = dt == KS_DTYPE_BF16;
+    const int ssg = (d + kSsGroup - 1) / kSsGroup;
     cudaStream_t s = m->stream;
     auto cap_ptr = [&](int plane) -> float* {
         if (capture_slot < 0) return nullptr;
         return hist_plane(m, plane) + (size_t)capture_slot * c.max_rows * d;
     };
+    auto runs = [&](int i) { return !mask || mask[i - 1]; };  // 1-based sublayer i
+    // gain of the RMSNorm that reads the residual after sublayer i (0 = embed):
+    // the next sublayer that runs, else the final norm
+    auto next_gain = [&](int i) -> const void* {
+        for (int k = i + 1; k <= 2 * c.n_layers; ++k)
+            if (runs(k)) return (k % 2 == 1) ? m->attn_norm[(k - 1) / 2] : m->mlp_norm[(k - 1) / 2];
+        return m->final_norm;
+    };
+    // input of a normalised projection
+    auto norm_input = [&](GemvArgs& g, const void* gain) {
+        g.ss_in = m->ss;
+        g.ss_groups = ssg;
+        g.eps = c.rms_eps;
+        if (bf) {
+            g.in = m->xg;       // x * gain in bf16, scaled by 1 / rms in the epilogue
+            g.in_ld = d;
+        } else {
+            g.in = m->x;        // fp32 kernel normalises while staging
+            g.in_ld = d;
+            g.norm_gain = gain;
+        }
+    };
+    auto resid_output = [&](GemvArgs& g, int after) {
+        g.resid = m->x;
+        g.resid_ld = d;
+        g.ss_out = m->ss;
+        g.capture = cap_ptr(after);
+        g.capture_ld = d;
+        if (bf) {
+            g.xg_out = m->xg;
+            g.next_gain = next_gain(after);
+        }
+    };
+    auto common = [&](GemvArgs& g, const void* W, int N, int K) {
+        g.W = W;
+        g.dtype = dt;
+        g.N = N;
+        g.K = K;
+        g.R = R;
+        g.partial = m->gemv_part;
+        g.counters = m->counters;
+        g.err = m->err;
+    };
     KS_TRY(launch(m, K_EMBED, [&]() -> cudaError_t {
-        if (dt == KS_DTYPE_BF16)
-            embed_kernel<__nv_bfloat16><<<R, 256, 0, s>>>(reinterpret_cast<const __nv_bfloat16*>(m->embed), tok, d,
-                                                           c.vocab, m->x, cap_ptr(0));
+        if (bf)
+            embed_kernel<__nv_bfloat16><<<R, 256, 0, s>>>(
+                reinterpret_cast<const __nv_bfloat16*>(m->embed), tok, d, c.vocab, m->x, cap_ptr(0), m->ss, m->xg,
+                reinterpret_cast<const __nv_bfloat16*>(next_gain(0)));
         else
             embed_kernel<float><<<R, 256, 0, s>>>(reinterpret_cast<const float*>(m->embed), tok, d, c.vocab, m->x,
-                                                  cap_ptr(0));
+                                                  cap_ptr(0), m->ss, nullptr, nullptr);
         return cudaGetLastError();
     }, "embed"));
 
     for (int l = 0; l < c.n_layers; ++l) {
-        const bool run_attn = !mask || mask[2 * l];
-        const bool run_mlp = !mask || mask[2 * l + 1];
+        const bool run_attn = runs(2 * l + 1);
+        const bool run_mlp = runs(2 * l + 2);
+        if ((!run_attn || !run_mlp) && capture_slot >= 0) {
+            set_error("forward: capture needs every sublayer");
+            return KS_ERR_STATE;
+        }
         if (run_attn) {
             GemvArgs g{};
-            g.W = m->w_qkv[l]; g.N = nqkv; g.K = d; g.R = R;
-            g.in = m->x; g.in_ld = d; g.norm_gain = m->attn_norm[l]; g.eps = c.rms_eps;
-            g.out = m->qkv; g.out_ld = nqkv;
-            g.partial = m->gemv_part; g.counters = m->counters;
+            common(g, m->w_qkv[l], nqkv, d);
+            norm_input(g, m->attn_norm[l]);
+            if (bf) { g.wmap = m->map_qkv[l]; g.xmap = m->map_xg[R > 8]; }
+            g.out = m->qkv;
+            g.out_ld = nqkv;
             gemv_plan(g, EPI_STORE);
             KS_TRY(launch(m, K_QKV, [&] { return launch_gemv(dt, EPI_STORE, g, s); }, "qkv"));
 
@@ -304,46 +381,44 @@ static ks_status forward(ks_model* m, const int32_t* tok, int R, int p0, const u
             KS_TRY(launch(m, K_MERGE, [&] { return launch_attn_merge(dt, at, s); }, "attention merge"));
 
             GemvArgs o{};
-            o.W = m->w_o[l]; o.N = d; o.K = c.n_q_heads * hd; o.R = R;
-            o.in = m->attn_out; o.in_ld = c.n_q_heads * hd;
-            o.resid = m->x; o.resid_ld = d;
-            o.capture = cap_ptr(2 * l + 1); o.capture_ld = d;
-            o.partial = m->gemv_part; o.counters = m->counters;
+            common(o, m->w_o[l], d, c.n_q_heads * hd);
+            if (bf) { o.wmap = m->map_o[l]; o.xmap = m->map_attn_out[R > 8]; }
+            o.in = m->attn_out;
+            o.in_ld = c.n_q_heads * hd;
+            resid_output(o, 2 * l + 1);
             gemv_plan(o, EPI_RESID);
             KS_TRY(launch(m, K_OPROJ, [&] { return launch_gemv(dt, EPI_RESID, o, s); }, "o-proj"));
-        } else if (capture_slot >= 0) {
-            set_error("forward: capture needs every sublayer");
-            return KS_ERR_STATE;
         }
         if (run_mlp) {
             GemvArgs gu{};
-            gu.W = m->w_gate_up[l]; gu.N = c.d_ff; gu.K = d; gu.R = R;
-            gu.in = m->x; gu.in_ld = d; gu.norm_gain = m->mlp_norm[l]; gu.eps = c.rms_eps;
-            gu.act = m->act; gu.act_ld = c.d_ff;
-            gu.partial = m->gemv_part; gu.counters = m->counters;
+            common(gu, m->w_gate_up[l], c.d_ff, d);
+            norm_input(gu, m->mlp_norm[l]);
+            if (bf) { gu.wmap = m->map_gu[l]; gu.xmap = m->map_xg[R > 8]; }
+            gu.act = m->act;
+            gu.act_ld = c.d_ff;
             gemv_plan(gu, EPI_SWIGLU);
             KS_TRY(launch(m, K_GATEUP, [&] { return launch_gemv(dt, EPI_SWIGLU, gu, s); }, "gate-up"));
 
             GemvArgs dn{};
-            dn.W = m->w_down[l]; dn.N = d; dn.K = c.d_ff; dn.R = R;
-            dn.in = m->act; dn.in_ld = c.d_ff;
-            dn.resid = m->x; dn.resid_ld = d;
-            dn.capture = cap_ptr(2 * l + 2); dn.capture_ld = d;
-            dn.partial = m->gemv_part; dn.counters = m->counters;
+            common(dn, m->w_down[l], d, c.d_ff);
+            if (bf) { dn.wmap = m->map_down[l]; dn.xmap = m->map_act[R > 8]; }
+            dn.in = m->act;
+            dn.in_ld = c.d_ff;
+            resid_output(dn, 2 * l + 2);
             gemv_plan(dn, EPI_RESID);
             KS_TRY(launch(m, K_DOWN, [&] { return launch_gemv(dt, EPI_RESID, dn, s); }, "down"));
-        } else if (capture_slot >= 0) {
-            set_error("forward: capture needs every sublayer");
-            return KS_ERR_STATE;
         }
     }
     if (argmax) {
         GemvArgs lm{};
-        lm.W = m->lm_head; lm.N = c.vocab; lm.K = d; lm.R = R;
-        lm.in = m->x; lm.in_ld = d; lm.norm_gain = m->final_norm; lm.eps = c.rms_eps;
-        lm.logits = m->logits; lm.logits_ld = c.vocab;
-        lm.amax_val = m->amax_val; lm.amax_idx = m->amax_idx; lm.tokens = argmax;
-        lm.counters = m->counters;
+        common(lm, m->lm_head, c.vocab, d);
+        norm_input(lm, m->final_norm);
+        if (bf) { lm.wmap = m->map_lm; lm.xmap = m->map_xg[R > 8]; }
+        lm.logits = m->logits;
+        lm.logits_ld = c.vocab;
+        lm.amax_val = m->amax_val;
+        lm.amax_idx = m->amax_idx;
+        lm.tokens = argmax;
         gemv_plan(lm, EPI_LMHEAD);
         KS_TRY(launch(m, K_LMHEAD, [&] { return launch_gemv(dt, EPI_LMHEAD, lm, s); }, "lm-head"));
     }
@@ -351,9 +426,18 @@ static ks_status forward(ks_model* m, const int32_t* tok, int R, int p0, const u
     return KS_OK;
 }
 
+// Wait for the stream, then read the device status word (set when a kernel's
+// bounded wait on an asynchronous copy gave up).
 static ks_status sync(ks_model* m, const char* what) {
-    cudaError_t e = cudaStreamSynchronize(m->stream);
+    int32_t* hs = m->h_buf + m->h_buf_ints - 1;
+    cudaError_t e = cudaMemcpyAsync(hs, m->err, sizeof(int32_t), cudaMemcpyDeviceToHost, m->stream);
     if (e != cudaSuccess) return cuda_fail(e, what);
+    e = cudaStreamSynchronize(m->stream);
+    if (e != cudaSuccess) return cuda_fail(e, what);
+    if (*hs != 0) {
+        set_error("%s: a kernel gave up waiting for an asynchronous copy", what);
+        return KS_ERR_TIMEOUT;
+    }
     return KS_OK;
 }
 
@@ -446,6 +530,8 @@ ks_status ks_model_create(const ks_config* cfg, const ks_weights* w, void* works
     m->kv = b + lay.kv;
     m->rope = reinterpret_cast<float*>(b + lay.rope);
     m->x = reinterpret_cast<float*>(b + lay.x);
+    m->ss = reinterpret_cast<float*>(b + lay.ss);
+    m->xg = reinterpret_cast<__nv_bfloat16*>(b + lay.xg);
     m->qkv = reinterpret_cast<float*>(b + lay.qkv);
     m->attn_out = b + lay.attn_out;
     m->act = b + lay.act;
@@ -460,6 +546,7 @@ ks_status ks_model_create(const ks_config* cfg, const ks_weights* w, void* works
     m->rows = tok;
     m->target = tok + (R + 1);
     m->result = tok + (2 * R + 1);
+    m->err = tok + (3 * R + 4);
     m->seq = tok + (3 * R + 8);
     m->hist = reinterpret_cast<float*>(b + lay.hist);
     m->hist_idx = reinterpret_cast<int*>(b + lay.hist_idx);
@@ -470,6 +557,32 @@ ks_status ks_model_create(const ks_config* cfg, const ks_weights* w, void* works
     m->select = b + lay.select;
     m->slot_off.assign(lay.hist_slots, 0);
     m->slot_cnt.assign(lay.hist_slots, 0);
+    if (m->dtype == KS_DTYPE_BF16) {
+        const int d = cfg->d_model, F = cfg->d_ff, hqd = cfg->n_q_heads * cfg->head_dim;
+        const int nqkv = (cfg->n_q_heads + 2 * cfg->n_kv_heads) * cfg->head_dim;
+        bool ok = true;
+        m->map_qkv.resize(L);
+        m->map_o.resize(L);
+        m->map_gu.resize(L);
+        m->map_down.resize(L);
+        for (int l = 0; l < L && ok; ++l) {
+            ok = ok && make_tma_map(&m->map_qkv[l], m->w_qkv[l], nqkv, d, 16);
+            ok = ok && make_tma_map(&m->map_o[l], m->w_o[l], d, hqd, 16);
+            ok = ok && make_tma_map(&m->map_gu[l], m->w_gate_up[l], 2 * (uint64_t)F, d, 16);
+            ok = ok && make_tma_map(&m->map_down[l], m->w_down[l], d, F, 16);
+        }
+        ok = ok && make_tma_map(&m->map_lm, m->lm_head, cfg->vocab, d, 16);
+        for (int b = 0; b < 2; ++b) {
+            ok = ok && make_tma_map(&m->map_xg[b], m->xg, R, d, 8u << b);
+            ok = ok && make_tma_map(&m->map_attn_out[b], m->attn_out, R, hqd, 8u << b);
+            ok = ok && make_tma_map(&m->map_act[b], m->act, R, F, 8u << b);
+        }
+        if (!ok) {
+            set_error("ks_model_create: TMA descriptor encoding failed");
+            delete m;
+            return KS_ERR_CUDA;
+        }
+    }
 
     auto fail = [&](cudaError_t e, const char* what) {
         ks_status st = cuda_fail(e, what);
@@ -503,7 +616,7 @@ ks_status ks_model_create(const ks_config* cfg, const ks_weights* w, void* works
     }
     e = cudaMemsetAsync(m->counters, 0, sizeof(int) * lay.counters_n, m->stream);
     if (e != cudaSuccess) return fail(e, "counter reset");
-    e = cudaMemsetAsync(b + lay.tok, 0, sizeof(int) * ((size_t)3 * R + 8 + cfg->max_seq), m->stream);
+    e = cudaMemsetAsync(b + lay.tok, 0, sizeof(int) * ((size_t)3 * R + 8 + cfg->max_seq), m->stream);  // incl. err
     if (e != cudaSuccess) return fail(e, "token reset");
     e = cudaStreamSynchronize(m->stream);
     if (e != cudaSuccess) return fail(e, "create sync");

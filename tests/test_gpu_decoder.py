@@ -4,9 +4,10 @@ against the oracle, plus the lossless invariant on the GPU itself.
 * Tiny fp32 workload (4 layers, 256-token prompt, 32 tokens, gamma 4): logits
   within 1e-4 relative, tokens equal to the oracle's wherever the oracle's
   top-2 margin exceeds 1e-3.
-* Small bf16 models (ragged d_ff, 300-token prompts spanning three attention
-  chunks, QK-norm on and off, head_dim 64 and 128): logits within 2e-2
-  relative (the workload tolerance), tokens under the same margin rule.
+* Small bf16 models (ragged d_ff 1368 = 85.5 x 16 and vocabulary 2000 =
+  31 x 64 + 16, 300-token prompts spanning three attention chunks, QK-norm on
+  and off, head_dim 64 and 128): logits within 2e-2 relative (the workload
+  tolerance), tokens under the same margin rule.
 * Lossless (Sec. 2.1): speculative output is bit-identical to the GPU's own
   greedy decode for every mask and the knapsack policy; a full-mask draft
   reproduces the target's logits bit for bit."""
@@ -27,7 +28,7 @@ def _gpu():
 
 def small_bf16(hd=128, qk_norm=False, L=2):
     from paper_2602_20217_gb300.configs import ModelShape
-    return ModelShape(f"small-bf16-hd{hd}", L, 512, 8, 2, hd, 1368, 2048, qk_norm=qk_norm,
+    return ModelShape(f"small-bf16-hd{hd}", L, 512, 8, 2, hd, 1368, 2000, qk_norm=qk_norm,
                       dtype="bf16", rope_theta=500000.0)
 
 
