@@ -1,22 +1,23 @@
 // Causal GQA attention over the KV cache for R <= 16 query rows (the Attn
 // sublayer of Sec. 2 inside a draft step or the gamma+1-row verify pass).
 //
-// Split-KV ("flash-decode"): one CTA per (KV head, chunk of kAttnChunk keys).
-// Chunk boundaries are absolute key positions and each chunk is split into
-// four fixed 32-key warp ranges merged in warp order, so the arithmetic
-// applied to one query row does not depend on how many rows share the pass:
-// keys past a row's own position are masked to -inf (their exp2 is exactly 0)
-// and chunks past it are skipped by the merge.  Greedy decoding and the
-// verify pass therefore produce bit-identical attention outputs.
+// Split-KV ("flash-decode") over a fixed partition of the key axis into
+// chunks whose boundaries are absolute positions (attn_chunk_start): 128 keys
+// below 8192, 512 keys below 32768, 2048 keys beyond.  One CTA per (KV head,
+// chunk); the largest chunks are scheduled first.  Keys past a row's own
+// position are masked to -inf (their exp2 is exactly 0) and chunks past it are
+// skipped by the merge, so the arithmetic applied to one query row does not
+// depend on how many rows share the pass: greedy decoding and the verify pass
+// produce bit-identical attention outputs.
 //
 // Per CTA: the new rows' K (QK-RMSNorm, RoPE) and V are written to the cache
-// by the CTA whose chunk holds their position, the G x R query vectors are
-// normalised, rotated and pre-scaled by log2(e)/sqrt(hd); K/V of the chunk are
-// staged in shared memory with cp.async (zero-filled past the valid keys).
-// bf16 models: S = Q K^T and O += P V on mma.sync.m16n8k16 with fp32 online
-// softmax in the log2 domain.  fp32 models: CUDA-core dot products.
-// Partials (m, l, o) per (row, query head, chunk) are merged by
-// attn_merge_kernel in a fixed order.
+// by the CTA whose chunk holds their position; the G x R query vectors are
+// normalised, rotated and pre-scaled by log2(e)/sqrt(hd).  bf16 models: K/V
+// tiles of 64 keys are double-buffered in shared memory with cp.async; each
+// warp owns a 16-row query tile and runs S = Q K^T and O += P V on
+// mma.sync.m16n8k16 with an fp32 online softmax in the log2 domain over the
+// whole chunk.  fp32 models: CUDA-core dot products.  Partials (m, l, o) per
+// (row, query head, chunk) are merged by attn_merge_kernel in a fixed order.
 #include "common.cuh"
 #include "internal.h"
 
@@ -24,7 +25,21 @@ namespace ks {
 
 constexpr int kAttnWarps = 4;
 constexpr int kPartPad = 4;  // partial row: m, l, 2 pad, o[hd] (16-byte aligned o)
+constexpr int kKeyTile = 64;
 constexpr float kLog2e = 1.4426950408889634f;
+
+// ------------------------------------------------------------ chunk schedule
+__host__ __device__ int attn_chunk_start(int c) {
+    if (c < 64) return 128 * c;
+    if (c < 112) return 8192 + 512 * (c - 64);
+    return 32768 + 2048 * (c - 112);
+}
+__host__ __device__ int attn_chunk_of(int pos) {
+    if (pos < 8192) return pos / 128;
+    if (pos < 32768) return 64 + (pos - 8192) / 512;
+    return 112 + (pos - 32768) / 2048;
+}
+int attn_num_chunks(int n_keys) { return n_keys <= 0 ? 0 : attn_chunk_of(n_keys - 1) + 1; }
 
 // ------------------------------------------------------------ small helpers
 KS_DEV void cp_async16(void* smem, const void* gmem, bool valid) {
@@ -32,7 +47,9 @@ KS_DEV void cp_async16(void* smem, const void* gmem, bool valid) {
     const int n = valid ? 16 : 0;
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(s), "l"(gmem), "r"(n));
 }
-KS_DEV void cp_async_wait_all() { asm volatile("cp.async.wait_all;\n" ::); }
+KS_DEV void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
+template <int N>
+KS_DEV void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N)); }
 
 KS_DEV void ldmatrix_x4(uint32_t (&r)[4], const void* p) {
     const uint32_t s = (uint32_t)__cvta_generic_to_shared(p);
@@ -47,7 +64,7 @@ KS_DEV void ldmatrix_x4_trans(uint32_t (&r)[4], const void* p) {
                  : "r"(s));
 }
 
-// Load one head vector (hd = 32 * NPL elements) of row r from the fp32
+// Load one head vector (hd = 32 * NPL elements) of a row from the fp32
 // projections, apply optional RMSNorm with gain, then rotate-half RoPE at
 // position pos.  Lane l holds elements l + 32 i.
 template <typename WT, int NPL>
@@ -77,256 +94,324 @@ KS_DEV void head_vector(const float* src, const WT* gain, float eps, const float
     }
 }
 
-// Prologue shared by both kernels: write this chunk's new K/V rows to the
-// cache and return the valid key range [cs, ce).
-template <typename WT, int NPL>
-KS_DEV void write_new_kv(const AttnArgs& a, int h, int cs, int ce) {
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+// Batched form of head_vector: a warp loads B vectors (and their RoPE rows) in
+// one round of independent loads, then normalises and rotates them.  valid[j]
+// = false skips vector j (its output is undefined).
+template <typename WT, int NPL, int B>
+KS_DEV void head_vectors(const float* const (&src)[B], const bool (&valid)[B], const int (&pos)[B],
+                         const WT* gain, float eps, const float* rope, float (&v)[B][NPL]) {
+    const int lane = threadIdx.x & 31;
     constexpr int hd = 32 * NPL;
-    WT* kc = reinterpret_cast<WT*>(a.kcache) + (size_t)h * a.max_seq * hd;
-    WT* vc = reinterpret_cast<WT*>(a.vcache) + (size_t)h * a.max_seq * hd;
-    const WT* kn = reinterpret_cast<const WT*>(a.k_norm);
-    for (int r = warp; r < a.R; r += kAttnWarps) {
-        const int pos = a.p0 + r;
-        if (pos < cs || pos >= ce) continue;
-        const float* row = a.qkv + (size_t)r * a.qkv_ld;
-        float k[NPL];
-        head_vector<WT, NPL>(row + (a.hq + h) * hd, kn, a.eps, a.rope, pos, k);
-        const float* vsrc = row + (a.hq + a.hk + h) * hd;
+    float cs[B][NPL / 2], sn[B][NPL / 2];
 #pragma unroll
-        for (int i = 0; i < NPL; ++i) {
-            kc[(size_t)pos * hd + lane + 32 * i] = from_float<WT>(k[i]);
-            vc[(size_t)pos * hd + lane + 32 * i] = from_float<WT>(vsrc[lane + 32 * i]);
+    for (int j = 0; j < B; ++j) {
+        if (!valid[j]) continue;
+#pragma unroll
+        for (int i = 0; i < NPL; ++i) v[j][i] = src[j][lane + 32 * i];
+        const float* rp = rope + (size_t)pos[j] * hd;
+#pragma unroll
+        for (int i = 0; i < NPL / 2; ++i) {
+            cs[j][i] = rp[2 * (lane + 32 * i)];
+            sn[j][i] = rp[2 * (lane + 32 * i) + 1];
+        }
+    }
+#pragma unroll
+    for (int j = 0; j < B; ++j) {
+        float ss = 0.f;
+        if (valid[j] && gain != nullptr) {
+#pragma unroll
+            for (int i = 0; i < NPL; ++i) ss = fmaf(v[j][i], v[j][i], ss);
+        }
+        if (gain != nullptr) ss = warp_sum(ss);  // every lane takes part (valid is warp-uniform)
+        if (!valid[j]) continue;
+        if (gain != nullptr) {
+            const float inv = rsqrtf(ss / (float)hd + eps);
+#pragma unroll
+            for (int i = 0; i < NPL; ++i) v[j][i] = (v[j][i] * inv) * to_float(gain[lane + 32 * i]);
+        }
+#pragma unroll
+        for (int i = 0; i < NPL / 2; ++i) {
+            const float a = v[j][i], b = v[j][i + NPL / 2];
+            v[j][i] = a * cs[j][i] - b * sn[j][i];
+            v[j][i + NPL / 2] = b * cs[j][i] + a * sn[j][i];
         }
     }
 }
 
+// Write this chunk's new K/V rows (positions p0 .. p0+R-1 inside [cs, ce)).
+template <typename WT, int NPL>
+KS_DEV void write_new_kv(const AttnArgs& a, int h, int cs, int ce) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    constexpr int hd = 32 * NPL;
+    constexpr int B = 4;
+    WT* kc = reinterpret_cast<WT*>(a.kcache) + (size_t)h * a.max_seq * hd;
+    WT* vc = reinterpret_cast<WT*>(a.vcache) + (size_t)h * a.max_seq * hd;
+    const WT* kn = reinterpret_cast<const WT*>(a.k_norm);
+    for (int r0 = warp * B; r0 < a.R; r0 += kAttnWarps * B) {
+        const float* src[B];
+        bool valid[B];
+        int pos[B];
+#pragma unroll
+        for (int j = 0; j < B; ++j) {
+            const int r = r0 + j;
+            pos[j] = a.p0 + r;
+            valid[j] = r < a.R && pos[j] >= cs && pos[j] < ce;
+            src[j] = a.qkv + (size_t)(valid[j] ? r : 0) * a.qkv_ld + (a.hq + h) * hd;
+            if (!valid[j]) pos[j] = 0;
+        }
+        float k[B][NPL];
+        head_vectors<WT, NPL, B>(src, valid, pos, kn, a.eps, a.rope, k);
+#pragma unroll
+        for (int j = 0; j < B; ++j) {
+            if (!valid[j]) continue;
+            const float* vsrc = a.qkv + (size_t)(r0 + j) * a.qkv_ld + (a.hq + a.hk + h) * hd;
+#pragma unroll
+            for (int i = 0; i < NPL; ++i) {
+                kc[(size_t)pos[j] * hd + lane + 32 * i] = from_float<WT>(k[j][i]);
+                vc[(size_t)pos[j] * hd + lane + 32 * i] = from_float<WT>(vsrc[lane + 32 * i]);
+            }
+        }
+    }
+}
+
+// chunk handled by this CTA: the largest (latest) chunks get the lowest blockIdx.y
+KS_DEV int my_chunk(const AttnArgs& a) {
+    const int nch = attn_chunk_of(a.p0 + a.R - 1) + 1;
+    return nch - 1 - (int)blockIdx.y;
+}
+
 // ----------------------------------------------------------- bf16 kernel
 // Shared layout (bf16, row pitch hd + 8 elements = 16 B padding):
-//   Qs [mpad][P]  Ks [C][P]  Vs [C][P]   then fp32 warp partials.
+//   Qs [mpad][P], then 2 stages of { Ks [64][P], Vs [64][P] }.
 template <int HD>
 __global__ void __launch_bounds__(128) attn_bf16_kernel(const AttnArgs a) {
     constexpr int NPL = HD / 32;
     constexpr int P = HD + 8;
-    constexpr int C = kAttnChunk;
-    constexpr int KW = C / kAttnWarps;  // keys per warp (32)
-    constexpr int NDT = HD / 8;         // dim tiles of 8
+    constexpr int NDT = HD / 8;  // dim tiles of 8
+    constexpr int KT = kKeyTile;
     extern __shared__ __align__(16) unsigned char smem[];
 
-    const int h = blockIdx.x, c = blockIdx.y;
+    const int h = blockIdx.x, c = my_chunk(a);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int g = lane >> 2, t = lane & 3;
     const int G = a.hq / a.hk;
     const int M = G * a.R;
     const int mtiles = (M + 15) >> 4;
     const int mpad = mtiles * 16;
-    const int cs = c * C;
-    const int ce = min(cs + C, a.p0 + a.R);
+    const int cs = attn_chunk_start(c);
+    const int ce = min(attn_chunk_start(c + 1), a.p0 + a.R);  // valid keys [cs, ce)
+    const int ntiles = (ce - cs + KT - 1) / KT;
 
     __nv_bfloat16* Qs = reinterpret_cast<__nv_bfloat16*>(smem);
-    __nv_bfloat16* Ks = Qs + (size_t)mpad * P;
-    __nv_bfloat16* Vs = Ks + (size_t)C * P;
-    float* wpart = reinterpret_cast<float*>(Vs + (size_t)C * P);  // [4][16][HD + 2] (m, l, o)
+    __nv_bfloat16* KV = Qs + (size_t)mpad * P;  // stage s: K at KV + s*2*KT*P, V after it
 
     // 1. new K/V rows of this chunk -> cache (generic stores, then barrier)
     write_new_kv<__nv_bfloat16, NPL>(a, h, cs, ce);
     __syncthreads();
 
-    // 2. stage K/V of keys [cs, ce) (zero past ce)
-    const __nv_bfloat16* kg = reinterpret_cast<const __nv_bfloat16*>(a.kcache) + ((size_t)h * a.max_seq + cs) * HD;
-    const __nv_bfloat16* vg = reinterpret_cast<const __nv_bfloat16*>(a.vcache) + ((size_t)h * a.max_seq + cs) * HD;
-    constexpr int CPR = HD / 8;  // 16-byte chunks per row
-    for (int i = tid; i < C * CPR; i += blockDim.x) {
-        const int row = i / CPR, col = (i - row * CPR) * 8;
-        const bool ok = cs + row < ce;
-        const size_t off = ok ? (size_t)row * HD + col : 0;
-        cp_async16(Ks + row * P + col, kg + off, ok);
-        cp_async16(Vs + row * P + col, vg + off, ok);
-    }
+    const __nv_bfloat16* kg = reinterpret_cast<const __nv_bfloat16*>(a.kcache) + (size_t)h * a.max_seq * HD;
+    const __nv_bfloat16* vg = reinterpret_cast<const __nv_bfloat16*>(a.vcache) + (size_t)h * a.max_seq * HD;
+    constexpr int CPR = HD / 8;  // 16-byte pieces per row
+    auto load_tile = [&](int ti) {
+        __nv_bfloat16* Ks = KV + (size_t)(ti & 1) * 2 * KT * P;
+        __nv_bfloat16* Vs = Ks + (size_t)KT * P;
+        const int k0 = cs + ti * KT;
+        for (int i = tid; i < KT * CPR; i += blockDim.x) {
+            const int row = i / CPR, col = (i - row * CPR) * 8;
+            const bool ok = k0 + row < ce;
+            const size_t off = ok ? (size_t)(k0 + row) * HD + col : 0;
+            cp_async16(Ks + row * P + col, kg + off, ok);
+            cp_async16(Vs + row * P + col, vg + off, ok);
+        }
+        cp_async_commit();
+    };
+    load_tile(0);
 
-    // 3. queries: m = r * G + gq, scaled into the log2 domain, bf16
+    // 2. queries: m = r * G + gq, scaled into the log2 domain, bf16
     const float qscale = kLog2e * rsqrtf((float)HD);
     const __nv_bfloat16* qn = reinterpret_cast<const __nv_bfloat16*>(a.q_norm);
-    for (int m = warp; m < mpad; m += kAttnWarps) {
-        if (m < M) {
-            const int r = m / G, gq = m - r * G;
-            float q[NPL];
-            head_vector<__nv_bfloat16, NPL>(a.qkv + (size_t)r * a.qkv_ld + (h * G + gq) * HD, qn, a.eps,
-                                            a.rope, a.p0 + r, q);
+    constexpr int QB = 4;
+    for (int m0 = warp * QB; m0 < mpad; m0 += kAttnWarps * QB) {
+        const float* src[QB];
+        bool valid[QB];
+        int pos[QB];
 #pragma unroll
-            for (int i = 0; i < NPL; ++i) Qs[m * P + lane + 32 * i] = __float2bfloat16_rn(q[i] * qscale);
-        } else {
+        for (int j = 0; j < QB; ++j) {
+            const int m = m0 + j;
+            valid[j] = m < M;
+            const int r = valid[j] ? m / G : 0, gq = valid[j] ? m - r * G : 0;
+            src[j] = a.qkv + (size_t)r * a.qkv_ld + (h * G + gq) * HD;
+            pos[j] = a.p0 + r;
+        }
+        float q[QB][NPL];
+        head_vectors<__nv_bfloat16, NPL, QB>(src, valid, pos, qn, a.eps, a.rope, q);
 #pragma unroll
-            for (int i = 0; i < NPL; ++i) Qs[m * P + lane + 32 * i] = __float2bfloat16_rn(0.f);
+        for (int j = 0; j < QB; ++j) {
+            const int m = m0 + j;
+            if (m >= mpad) continue;
+#pragma unroll
+            for (int i = 0; i < NPL; ++i)
+                Qs[m * P + lane + 32 * i] = __float2bfloat16_rn(valid[j] ? q[j][i] * qscale : 0.f);
         }
     }
-    cp_async_wait_all();
-    __syncthreads();
 
-    const int kbase = warp * KW;  // warp's key range within the chunk
-    for (int mt = 0; mt < mtiles; ++mt) {
-        // Q fragments of this m-tile
+    // 3. rounds of up to four m-tiles (one per warp) over the chunk's key tiles
+    for (int mt0 = 0; mt0 < mtiles; mt0 += kAttnWarps) {
+        const int mt = mt0 + warp;
+        const bool active = mt < mtiles;
+        if (mt0 > 0) load_tile(0);  // a new round streams the chunk again
         uint32_t qf[HD / 16][4];
-#pragma unroll
-        for (int ks = 0; ks < HD / 16; ++ks) {
-            const int mi = lane >> 3;
-            const int row = mt * 16 + (mi & 1) * 8 + (lane & 7);
-            const int col = ks * 16 + (mi >> 1) * 8;
-            ldmatrix_x4(qf[ks], Qs + row * P + col);
-        }
-        // row positions of the two rows this thread holds
-        int rpos[2];
-#pragma unroll
-        for (int hh = 0; hh < 2; ++hh) {
-            const int m = mt * 16 + g + 8 * hh;
-            rpos[hh] = (m < M) ? a.p0 + m / G : -1;  // padding rows see no key
-        }
+        int rpos[2] = {-1, -1};
         float o[NDT][4];
-#pragma unroll
-        for (int i = 0; i < NDT; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
         float mrow[2] = {-INFINITY, -INFINITY};
         float lrow[2] = {0.f, 0.f};
+#pragma unroll
+        for (int i = 0; i < NDT; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
+        bool qloaded = false;
 
-        for (int kt = 0; kt < KW; kt += 16) {
-            const int key0 = kbase + kt;  // within chunk
-            // S = Q K^T for 16 keys (two n-tiles of 8)
-            float s[2][4];
-#pragma unroll
-            for (int j = 0; j < 2; ++j) s[j][0] = s[j][1] = s[j][2] = s[j][3] = 0.f;
-#pragma unroll
-            for (int ks = 0; ks < HD / 16; ++ks) {
-                uint32_t kb[4];
-                // matrices: (keys 0-7, d 0-7), (keys 0-7, d 8-15), (keys 8-15, d 0-7), (keys 8-15, d 8-15)
-                const int mi = lane >> 3;
-                const int krow = key0 + (mi >> 1) * 8 + (lane & 7);
-                const int kcol = ks * 16 + (mi & 1) * 8;
-                ldmatrix_x4(kb, Ks + krow * P + kcol);
-                mma_bf16(s[0], qf[ks][0], qf[ks][1], qf[ks][2], qf[ks][3], kb[0], kb[1]);
-                mma_bf16(s[1], qf[ks][0], qf[ks][1], qf[ks][2], qf[ks][3], kb[2], kb[3]);
+        for (int ti = 0; ti < ntiles; ++ti) {
+            if (ti + 1 < ntiles) {
+                load_tile(ti + 1);
+                cp_async_wait<1>();
+            } else {
+                cp_async_wait<0>();
             }
-            // causal / validity mask and online softmax (log2 domain)
+            __syncthreads();  // tile ti (and, first time, Qs) visible
+            if (active) {
+                if (!qloaded) {
 #pragma unroll
-            for (int hh = 0; hh < 2; ++hh) {
-                float tmax = -INFINITY;
-#pragma unroll
-                for (int j = 0; j < 2; ++j)
-#pragma unroll
-                    for (int e = 0; e < 2; ++e) {
-                        const int key = cs + key0 + j * 8 + 2 * t + e;
-                        float& v = s[j][2 * hh + e];
-                        if (key > rpos[hh] || key >= ce) v = -INFINITY;
-                        tmax = fmaxf(tmax, v);
+                    for (int ks = 0; ks < HD / 16; ++ks) {
+                        const int mi = lane >> 3;
+                        const int row = mt * 16 + (mi & 1) * 8 + (lane & 7);
+                        const int col = ks * 16 + (mi >> 1) * 8;
+                        ldmatrix_x4(qf[ks], Qs + row * P + col);
                     }
-                tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 1));
-                tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 2));
-                const float mnew = fmaxf(mrow[hh], tmax);
-                float alpha, psum = 0.f;
-                if (mnew == -INFINITY) {
-                    alpha = 1.f;
 #pragma unroll
-                    for (int j = 0; j < 2; ++j) s[j][2 * hh] = s[j][2 * hh + 1] = 0.f;
-                } else {
-                    alpha = exp2f(mrow[hh] - mnew);
+                    for (int hh = 0; hh < 2; ++hh) {
+                        const int m = mt * 16 + g + 8 * hh;
+                        rpos[hh] = (m < M) ? a.p0 + m / G : -1;  // padding rows see no key
+                    }
+                    qloaded = true;
+                }
+                const __nv_bfloat16* Ks = KV + (size_t)(ti & 1) * 2 * KT * P;
+                const __nv_bfloat16* Vs = Ks + (size_t)KT * P;
+                const int kbase = cs + ti * KT;
 #pragma unroll
-                    for (int j = 0; j < 2; ++j)
+                for (int kk = 0; kk < KT; kk += 16) {
+                    float s[2][4];
 #pragma unroll
-                        for (int e = 0; e < 2; ++e) {
-                            float& v = s[j][2 * hh + e];
-                            v = exp2f(v - mnew);
-                            psum += v;
+                    for (int j = 0; j < 2; ++j) s[j][0] = s[j][1] = s[j][2] = s[j][3] = 0.f;
+#pragma unroll
+                    for (int ks = 0; ks < HD / 16; ++ks) {
+                        uint32_t kb[4];
+                        const int mi = lane >> 3;
+                        const int krow = kk + (mi >> 1) * 8 + (lane & 7);
+                        const int kcol = ks * 16 + (mi & 1) * 8;
+                        ldmatrix_x4(kb, Ks + krow * P + kcol);
+                        mma_bf16(s[0], qf[ks][0], qf[ks][1], qf[ks][2], qf[ks][3], kb[0], kb[1]);
+                        mma_bf16(s[1], qf[ks][0], qf[ks][1], qf[ks][2], qf[ks][3], kb[2], kb[3]);
+                    }
+                    // causal / validity mask and online softmax (log2 domain)
+#pragma unroll
+                    for (int hh = 0; hh < 2; ++hh) {
+                        float tmax = -INFINITY;
+#pragma unroll
+                        for (int j = 0; j < 2; ++j)
+#pragma unroll
+                            for (int e = 0; e < 2; ++e) {
+                                const int key = kbase + kk + j * 8 + 2 * t + e;
+                                float& v = s[j][2 * hh + e];
+                                if (key > rpos[hh] || key >= ce) v = -INFINITY;
+                                tmax = fmaxf(tmax, v);
+                            }
+                        tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 1));
+                        tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 2));
+                        const float mnew = fmaxf(mrow[hh], tmax);
+                        float alpha, psum = 0.f;
+                        if (mnew == -INFINITY) {
+                            alpha = 1.f;
+#pragma unroll
+                            for (int j = 0; j < 2; ++j) s[j][2 * hh] = s[j][2 * hh + 1] = 0.f;
+                        } else {
+                            alpha = exp2f(mrow[hh] - mnew);
+#pragma unroll
+                            for (int j = 0; j < 2; ++j)
+#pragma unroll
+                                for (int e = 0; e < 2; ++e) {
+                                    float& v = s[j][2 * hh + e];
+                                    v = exp2f(v - mnew);
+                                    psum += v;
+                                }
                         }
-                }
-                mrow[hh] = mnew;
-                lrow[hh] = lrow[hh] * alpha + psum;
+                        mrow[hh] = mnew;
+                        lrow[hh] = lrow[hh] * alpha + psum;
 #pragma unroll
-                for (int i = 0; i < NDT; ++i) {
-                    o[i][2 * hh] *= alpha;
-                    o[i][2 * hh + 1] *= alpha;
+                        for (int i = 0; i < NDT; ++i) {
+                            o[i][2 * hh] *= alpha;
+                            o[i][2 * hh + 1] *= alpha;
+                        }
+                    }
+                    // O += P V
+                    const uint32_t pa0 = pack_bf16(s[0][0], s[0][1]);
+                    const uint32_t pa1 = pack_bf16(s[0][2], s[0][3]);
+                    const uint32_t pa2 = pack_bf16(s[1][0], s[1][1]);
+                    const uint32_t pa3 = pack_bf16(s[1][2], s[1][3]);
+#pragma unroll
+                    for (int dp = 0; dp < NDT / 2; ++dp) {
+                        uint32_t vb[4];
+                        const int mi = lane >> 3;
+                        const int vrow = kk + (mi & 1) * 8 + (lane & 7);
+                        const int vcol = dp * 16 + (mi >> 1) * 8;
+                        ldmatrix_x4_trans(vb, Vs + vrow * P + vcol);
+                        mma_bf16(o[2 * dp], pa0, pa1, pa2, pa3, vb[0], vb[1]);
+                        mma_bf16(o[2 * dp + 1], pa0, pa1, pa2, pa3, vb[2], vb[3]);
+                    }
                 }
             }
-            // O += P V
-            const uint32_t pa0 = pack_bf16(s[0][0], s[0][1]);
-            const uint32_t pa1 = pack_bf16(s[0][2], s[0][3]);
-            const uint32_t pa2 = pack_bf16(s[1][0], s[1][1]);
-            const uint32_t pa3 = pack_bf16(s[1][2], s[1][3]);
-#pragma unroll
-            for (int dp = 0; dp < NDT / 2; ++dp) {
-                uint32_t vb[4];
-                // matrices: (keys 0-7, d), (keys 8-15, d), (keys 0-7, d+8), (keys 8-15, d+8)
-                const int mi = lane >> 3;
-                const int vrow = key0 + (mi & 1) * 8 + (lane & 7);
-                const int vcol = dp * 16 + (mi >> 1) * 8;
-                ldmatrix_x4_trans(vb, Vs + vrow * P + vcol);
-                mma_bf16(o[2 * dp], pa0, pa1, pa2, pa3, vb[0], vb[1]);
-                mma_bf16(o[2 * dp + 1], pa0, pa1, pa2, pa3, vb[2], vb[3]);
-            }
+            __syncthreads();  // everyone is done with tile ti before it is refilled
         }
-        // full row sums of l across the quad
+        if (!active) continue;
+        // full row sums of l across the quad, then this chunk's partials
 #pragma unroll
         for (int hh = 0; hh < 2; ++hh) {
             lrow[hh] += __shfl_xor_sync(0xffffffffu, lrow[hh], 1);
             lrow[hh] += __shfl_xor_sync(0xffffffffu, lrow[hh], 2);
         }
-        // warp partials -> shared
-        float* wp = wpart + (size_t)warp * 16 * (HD + 2);
 #pragma unroll
         for (int hh = 0; hh < 2; ++hh) {
-            const int rr = g + 8 * hh;
+            const int m = mt * 16 + g + 8 * hh;
+            if (m >= M) continue;
+            const int r = m / G, gq = m - r * G;
+            float* dst = a.part + (((size_t)r * a.hq + h * G + gq) * a.n_chunks_max + c) * (HD + kPartPad);
             if (t == 0) {
-                wp[rr * (HD + 2) + 0] = mrow[hh];
-                wp[rr * (HD + 2) + 1] = lrow[hh];
+                dst[0] = mrow[hh];
+                dst[1] = lrow[hh];
             }
 #pragma unroll
             for (int i = 0; i < NDT; ++i) {
-                wp[rr * (HD + 2) + 2 + i * 8 + 2 * t] = o[i][2 * hh];
-                wp[rr * (HD + 2) + 2 + i * 8 + 2 * t + 1] = o[i][2 * hh + 1];
+                dst[kPartPad + i * 8 + 2 * t] = o[i][2 * hh];
+                dst[kPartPad + i * 8 + 2 * t + 1] = o[i][2 * hh + 1];
             }
         }
-        __syncthreads();
-        // merge the four warp ranges in warp order -> global chunk partial
-        for (int idx = tid; idx < 16 * (HD + 2); idx += blockDim.x) {
-            const int rr = idx / (HD + 2), col = idx - rr * (HD + 2);
-            const int m = mt * 16 + rr;
-            if (m >= M) continue;
-            float mx = -INFINITY;
-#pragma unroll
-            for (int w = 0; w < kAttnWarps; ++w) mx = fmaxf(mx, wpart[(size_t)w * 16 * (HD + 2) + rr * (HD + 2)]);
-            float out;
-            if (col == 0) {
-                out = mx;
-            } else if (mx == -INFINITY) {
-                out = 0.f;
-            } else {
-                out = 0.f;
-#pragma unroll
-                for (int w = 0; w < kAttnWarps; ++w) {
-                    const float* wpw = wpart + (size_t)w * 16 * (HD + 2) + rr * (HD + 2);
-                    const float mw = wpw[0];
-                    if (mw != -INFINITY) out += exp2f(mw - mx) * wpw[col];
-                }
-            }
-            const int r = m / G, gq = m - r * G;
-            float* dst = a.part + (((size_t)r * a.hq + h * G + gq) * a.n_chunks_max + c) * (HD + kPartPad);
-            dst[col < 2 ? col : col + 2] = out;
-        }
-        __syncthreads();
     }
 }
 
 // ----------------------------------------------------------- fp32 kernel
-// One warp per query row at a time; K/V read from the cache (L2).
+// One warp per query row at a time; K/V read from the cache (L2).  Used for
+// fp32 models.
 template <int HD>
 __global__ void __launch_bounds__(128) attn_f32_kernel(const AttnArgs a) {
     constexpr int NPL = HD / 32;
-    constexpr int C = kAttnChunk;
-    __shared__ float qsh[kAttnWarps][HD];
-    __shared__ float psh[kAttnWarps][C];
-    const int h = blockIdx.x, c = blockIdx.y;
+    constexpr int C = 2048;  // largest chunk of the schedule
+    extern __shared__ float fsm[];
+    float* qsh = fsm;                    // [4][HD]
+    float* psh = fsm + kAttnWarps * HD;  // [4][C]
+    const int h = blockIdx.x, c = my_chunk(a);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int G = a.hq / a.hk;
     const int M = G * a.R;
-    const int cs = c * C;
-    const int ce = min(cs + C, a.p0 + a.R);
+    const int cs = attn_chunk_start(c);
+    const int ce = min(attn_chunk_start(c + 1), a.p0 + a.R);
 
     write_new_kv<float, NPL>(a, h, cs, ce);
     __syncthreads();
@@ -335,33 +420,34 @@ __global__ void __launch_bounds__(128) attn_f32_kernel(const AttnArgs a) {
     const float* vc = reinterpret_cast<const float*>(a.vcache) + (size_t)h * a.max_seq * HD;
     const float qscale = kLog2e * rsqrtf((float)HD);
     const float* qn = reinterpret_cast<const float*>(a.q_norm);
+    float* q_w = qsh + warp * HD;
+    float* p_w = psh + warp * C;
     for (int m = warp; m < M; m += kAttnWarps) {
         const int r = m / G, gq = m - r * G;
         const int pos = a.p0 + r;
         float q[NPL];
         head_vector<float, NPL>(a.qkv + (size_t)r * a.qkv_ld + (h * G + gq) * HD, qn, a.eps, a.rope, pos, q);
 #pragma unroll
-        for (int i = 0; i < NPL; ++i) qsh[warp][lane + 32 * i] = q[i] * qscale;
+        for (int i = 0; i < NPL; ++i) q_w[lane + 32 * i] = q[i] * qscale;
         __syncwarp();
         const int kend = min(ce, pos + 1);
-        // scores: lane owns keys cs + lane + 32 j
         float mx = -INFINITY;
-        for (int j = lane; j < C; j += 32) {
+        for (int j = lane; j < ce - cs; j += 32) {
             const int key = cs + j;
             float sc = -INFINITY;
             if (key < kend) {
                 sc = 0.f;
                 const float* kr = kc + (size_t)key * HD;
-                for (int d = 0; d < HD; ++d) sc = fmaf(qsh[warp][d], kr[d], sc);
+                for (int d = 0; d < HD; ++d) sc = fmaf(q_w[d], kr[d], sc);
             }
-            psh[warp][j] = sc;
+            p_w[j] = sc;
             mx = fmaxf(mx, sc);
         }
         mx = warp_max(mx);
         float l = 0.f;
-        for (int j = lane; j < C; j += 32) {
-            const float p = (mx == -INFINITY || psh[warp][j] == -INFINITY) ? 0.f : exp2f(psh[warp][j] - mx);
-            psh[warp][j] = p;
+        for (int j = lane; j < ce - cs; j += 32) {
+            const float p = (mx == -INFINITY || p_w[j] == -INFINITY) ? 0.f : exp2f(p_w[j] - mx);
+            p_w[j] = p;
             l += p;
         }
         l = warp_sum(l);
@@ -369,7 +455,7 @@ __global__ void __launch_bounds__(128) attn_f32_kernel(const AttnArgs a) {
         float* dst = a.part + (((size_t)r * a.hq + h * G + gq) * a.n_chunks_max + c) * (HD + kPartPad);
         for (int d = lane; d < HD; d += 32) {
             float acc = 0.f;
-            for (int j = 0; j < kend - cs; ++j) acc = fmaf(psh[warp][j], vc[(size_t)(cs + j) * HD + d], acc);
+            for (int j = 0; j < kend - cs; ++j) acc = fmaf(p_w[j], vc[(size_t)(cs + j) * HD + d], acc);
             dst[kPartPad + d] = acc;
         }
         if (lane == 0) {
@@ -382,20 +468,20 @@ __global__ void __launch_bounds__(128) attn_f32_kernel(const AttnArgs a) {
 
 // ------------------------------------------------------------------ merge
 // out[r][hq_idx * hd + d] = sum_c 2^(m_c - M) o_c[d] / sum_c 2^(m_c - M) l_c over
-// the chunks 0 .. pos_r / C of row r.  Fixed order for every term: the max is
-// exact in any order; l and o are summed per thread (stride 128 over chunks)
-// or per warp (chunks c = w mod 4) and then in thread / warp order.  The
-// chunk count depends only on the row's position, so a row gives the same
-// bits in a 1-row pass and in a gamma+1-row pass.
+// the chunks 0 .. chunk_of(pos_r) of row r.  Fixed order for every term: the
+// max is exact in any order; l and o are summed per thread (stride 128 over
+// chunks) or per warp (chunks c = w mod 4) and then in thread / warp order.
+// The chunk count depends only on the row's position, so a row gives the
+// same bits in a 1-row pass and in a gamma+1-row pass.
 template <typename WT, int HD>
 __global__ void __launch_bounds__(128) attn_merge_kernel(const AttnArgs a) {
-    extern __shared__ float wsh[];           // [nch] chunk weights
+    extern __shared__ float wsh[];  // [nch] chunk weights
     __shared__ float red[kAttnWarps + 1];
     __shared__ float osh[kAttnWarps][HD];
     const int hq_idx = blockIdx.x, r = blockIdx.y;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int pos = a.p0 + r;
-    const int nch = pos / kAttnChunk + 1;
+    const int nch = attn_chunk_of(pos) + 1;
     constexpr int S = HD + kPartPad;
     const float* base = a.part + ((size_t)r * a.hq + hq_idx) * a.n_chunks_max * S;
     float mx = -INFINITY;
@@ -411,8 +497,8 @@ __global__ void __launch_bounds__(128) attn_merge_kernel(const AttnArgs a) {
         wsh[c] = w;
         ls = fmaf(w, base[(size_t)c * S + 1], ls);
     }
-    const float L = block_sum<kAttnWarps>(ls, red);   // ends with a barrier: wsh is visible
-    constexpr int PER = HD / 32;                      // dims per lane
+    const float L = block_sum<kAttnWarps>(ls, red);  // ends with a barrier: wsh is visible
+    constexpr int PER = HD / 32;                     // dims per lane
     float o[PER];
 #pragma unroll
     for (int i = 0; i < PER; ++i) o[i] = 0.f;
@@ -443,13 +529,12 @@ __global__ void __launch_bounds__(128) attn_merge_kernel(const AttnArgs a) {
 // --------------------------------------------------------------- launchers
 static size_t attn_bf16_smem(int HD, int mpad) {
     const int P = HD + 8;
-    return sizeof(__nv_bfloat16) * ((size_t)mpad * P + 2 * (size_t)kAttnChunk * P) +
-           sizeof(float) * kAttnWarps * 16 * (HD + 2);
+    return sizeof(__nv_bfloat16) * ((size_t)mpad * P + 2 * 2 * (size_t)kKeyTile * P);
 }
 
 cudaError_t launch_attention(int dtype, const AttnArgs& a, cudaStream_t s) {
-    const int nch = (a.p0 + a.R + kAttnChunk - 1) / kAttnChunk;
-    if (nch > a.n_chunks_max) return cudaErrorInvalidValue;
+    const int nch = attn_num_chunks(a.p0 + a.R);
+    if (nch > a.n_chunks_max || a.p0 + a.R > a.max_seq) return cudaErrorInvalidValue;
     dim3 grid(a.hk, nch);
     if (dtype == 1) {
         const int M = (a.hq / a.hk) * a.R;
@@ -465,15 +550,21 @@ cudaError_t launch_attention(int dtype, const AttnArgs& a, cudaStream_t s) {
         if (a.hd == 64) return run(attn_bf16_kernel<64>);
         return cudaErrorInvalidValue;
     }
-    if (a.hd == 128) attn_f32_kernel<128><<<grid, 128, 0, s>>>(a);
-    else if (a.hd == 64) attn_f32_kernel<64><<<grid, 128, 0, s>>>(a);
-    else return cudaErrorInvalidValue;
-    return cudaGetLastError();
+    const size_t smem = sizeof(float) * kAttnWarps * ((size_t)a.hd + 2048);
+    auto run = [&](auto kern) -> cudaError_t {
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        kern<<<grid, 128, smem, s>>>(a);
+        return cudaGetLastError();
+    };
+    if (a.hd == 128) return run(attn_f32_kernel<128>);
+    if (a.hd == 64) return run(attn_f32_kernel<64>);
+    return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_attn_merge(int dtype, const AttnArgs& a, cudaStream_t s) {
     dim3 grid(a.hq, a.R);
-    const int nch = (a.p0 + a.R - 1) / kAttnChunk + 1;
+    const int nch = attn_num_chunks(a.p0 + a.R);
     const size_t smem = sizeof(float) * (size_t)nch;
     if (smem > 48 * 1024) return cudaErrorInvalidValue;
     if (dtype == 1) {

@@ -386,8 +386,8 @@ __global__ void __launch_bounds__(128) gemv_f32_kernel(const GemvArgs a) {
 // ------------------------------------------------- bf16 streaming kernel
 // Work item = 16 output features (16 weight rows, or 16 gate + 16 up rows)
 // over the full K.  A ring stage holds NB x 256 columns of the item's weight
-// rows (one 256 x 16 TMA box per 256 columns and row block) and of its
-// activation rows (256 x 8 or 256 x 16 boxes), rows 512 bytes apart.  The four
+// rows (one 256 x 16 TMA box per 256 columns and row block) and of its R
+// activation rows (256 x R boxes), rows 512 bytes apart.  The four
 // consumer warps split each stage's columns evenly; at the end of an item
 // their partial fragments are added in warp order in shared memory.
 //
@@ -526,6 +526,8 @@ __global__ void __launch_bounds__(160, 1) gemv_stream_kernel(const __grid_consta
 #pragma unroll
             for (int b = 0; b < Cfg::kNB; ++b) tma_2d(st + b * Cfg::kBoxA, &a.xmap, k0 + 256 * b, 0, &full[slot]);
         };
+        // bytes landing per stage: the weight boxes plus activation boxes of R rows
+        const uint32_t bytes = 2u * (Cfg::kWBlocks * Cfg::kNB * Cfg::kBoxW + Cfg::kNB * 256 * a.R);
         // first item (static): weights before the grid dependency resolves
         int it = blockIdx.x;
         int t = 0;
@@ -533,7 +535,7 @@ __global__ void __launch_bounds__(160, 1) gemv_stream_kernel(const __grid_consta
         for (int kt = 0; kt < pre; ++kt) {
             slot_item[kt] = it;
             slot_kt[kt] = kt;
-            mbar_expect_tx(&full[kt], Cfg::kBytes);
+            mbar_expect_tx(&full[kt], bytes);
             load_w(kt, it, kt);
         }
         grid_dependency_wait();
@@ -551,7 +553,7 @@ __global__ void __launch_bounds__(160, 1) gemv_stream_kernel(const __grid_consta
                     }
                     slot_item[slot] = it;
                     slot_kt[slot] = kt;
-                    mbar_expect_tx(&full[slot], Cfg::kBytes);
+                    mbar_expect_tx(&full[slot], bytes);
                     load_w(slot, it, kt);
                     load_x(slot, kt);
                 }

@@ -15,7 +15,7 @@ enum GemvEpi { EPI_STORE = 0, EPI_RESID = 1, EPI_SWIGLU = 2, EPI_LMHEAD = 3 };
 
 struct GemvArgs {
     CUtensorMap wmap;       // bf16: TMA map of W (dims {K, rows}, box 256 x 16)
-    CUtensorMap xmap;       // bf16: TMA map of the input rows (dims {K, max_rows}, box 256 x 8 or 16)
+    CUtensorMap xmap;       // bf16: TMA map of the input rows (dims {K, max_rows}, box 256 x R)
     int dtype;              // KS_DTYPE_F32 / KS_DTYPE_BF16 (selects kernel and split plan)
     const void* W;          // [N (or 2N for SwiGLU)][K], row stride K, model dtype
     int N;                  // output features (SwiGLU: d_ff; rows n and N + n pair up)
@@ -68,7 +68,6 @@ struct AttnArgs {
     const void* q_norm;     // [hd] or null (model dtype)
     const void* k_norm;
     float eps;
-    int chunk;              // keys per CTA (fixed; split boundaries are absolute)
     float* part;            // [R][hq][n_chunks_max][hd + 4] (m, l, pad, pad, o[hd])
     int n_chunks_max;
     void* out;              // [R][hq hd] model dtype: merged attention output
@@ -77,7 +76,9 @@ struct AttnArgs {
 
 cudaError_t launch_attention(int dtype, const AttnArgs& a, cudaStream_t s);
 cudaError_t launch_attn_merge(int dtype, const AttnArgs& a, cudaStream_t s);
-constexpr int kAttnChunk = 128;
+// Fixed partition of the key axis for split-KV attention (absolute positions):
+// chunks of 128 keys below 8192, 512 below 32768, 2048 beyond.
+int attn_num_chunks(int n_keys);
 constexpr int kSsGroup = 16;    // features per sum-of-squares partial (= rows of a bf16 GEMV work item)
 
 // ---------------------------------------------------------------- select

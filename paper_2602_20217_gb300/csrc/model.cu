@@ -40,37 +40,30 @@ enum { K_QKV = 0, K_ATTN, K_MERGE, K_OPROJ, K_GATEUP, K_DOWN, K_LMHEAD, K_EMBED,
 
 // ------------------------------------------------------------ small kernels
 // x[r] = embed[tok[r]] (fp32); optionally copied to the history plane 0.
-// Also the per-64-feature sums of squares ss[g][r] that the next RMSNorm
-// uses (lane l adds features 64 g + l and 64 g + 32 + l, then a butterfly -
-// the same order as the residual epilogues).
+// Block (r, b) covers features [256 b, 256 b + 256) of row r; it also writes
+// the bf16 x * gain input of the next projection and the 16-feature sums of
+// squares ss[q][r] that its RMSNorm uses.
 template <typename WT>
-__global__ void embed_kernel(const WT* embed, const int32_t* tok, int d, int vocab, float* x,
-                             float* capture, float* ss, __nv_bfloat16* xg, const WT* next_gain) {
+__global__ void __launch_bounds__(256) embed_kernel(const WT* embed, const int32_t* tok, int d, int vocab, float* x,
+                                                    float* capture, float* ss, __nv_bfloat16* xg,
+                                                    const WT* next_gain) {
     const int r = blockIdx.x;
+    const int k = blockIdx.y * 256 + threadIdx.x;
     int t = tok[r];
     if (t < 0 || t >= vocab) t = 0;
-    const WT* e = embed + (size_t)t * d;
-    for (int k = threadIdx.x; k < d; k += blockDim.x) {
-        const float v = to_float(e[k]);
+    float v = 0.f;
+    if (k < d) {
+        v = to_float(embed[(size_t)t * d + k]);
         x[(size_t)r * d + k] = v;
         if (capture) capture[(size_t)r * d + k] = v;
         if (xg) xg[(size_t)r * d + k] = __float2bfloat16_rn(v * to_float(next_gain[k]));
     }
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int groups = (d + kSsGroup - 1) / kSsGroup;
-    // two 16-feature groups per warp pass: lanes 0-15 and 16-31
-    for (int gp = 2 * warp; gp < groups; gp += 2 * (blockDim.x / 32)) {
-        const int q = gp + (lane >> 4);
-        const int n = q * kSsGroup + (lane & 15);
-        float s = 0.f;
-        if (q < groups && n < d) {
-            const float v = to_float(e[n]);
-            s = v * v;
-        }
+    // lanes 0-15 and 16-31 of each warp form one 16-feature group
+    float s = v * v;
 #pragma unroll
-        for (int o = 8; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-        if ((lane & 15) == 0 && q < groups) ss[q * 16 + r] = s;
-    }
+    for (int o = 8; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    const int lane = threadIdx.x & 31;
+    if ((lane & 15) == 0 && k < d) ss[(k / kSsGroup) * 16 + r] = s;
 }
 
 // Greedy acceptance (Sec. 2.1): drafts = rows[1..gamma], z = target argmax of
@@ -123,7 +116,7 @@ static Layout make_layout(const ks_config* c) {
     const int d = c->d_model, hd = c->head_dim, R = c->max_rows;
     const int nqkv = (c->n_q_heads + 2 * c->n_kv_heads) * hd;
     const int nsub = 2 * c->n_layers;
-    L.n_chunks_max = (c->max_seq + kAttnChunk - 1) / kAttnChunk;
+    L.n_chunks_max = attn_num_chunks(c->max_seq);
     L.hist_slots = c->hist_steps + 1;
     size_t gp = 0;
     gp = std::max(gp, gemv_partial_floats(nqkv, d, R, EPI_STORE, c->dtype));
@@ -218,7 +211,7 @@ struct ks_model {
     int64_t h2d = 0, d2h = 0;
     // bf16: TMA maps of every weight matrix and of the three projection inputs
     std::vector<CUtensorMap> map_qkv, map_o, map_gu, map_down;
-    CUtensorMap map_lm, map_xg[2], map_attn_out[2], map_act[2];  // [0]: 8-row boxes, [1]: 16-row boxes
+    CUtensorMap map_lm, map_xg[16], map_attn_out[16], map_act[16];  // [R - 1]: boxes of exactly R rows
     KlassTiming timing[kKlasses];
 };
 
@@ -341,11 +334,11 @@ static ks_status forward(ks_model* m, const int32_t* tok, int R, int p0, const u
     };
     KS_TRY(launch(m, K_EMBED, [&]() -> cudaError_t {
         if (bf)
-            embed_kernel<__nv_bfloat16><<<R, 256, 0, s>>>(
+            embed_kernel<__nv_bfloat16><<<dim3(R, (d + 255) / 256), 256, 0, s>>>(
                 reinterpret_cast<const __nv_bfloat16*>(m->embed), tok, d, c.vocab, m->x, cap_ptr(0), m->ss, m->xg,
                 reinterpret_cast<const __nv_bfloat16*>(next_gain(0)));
         else
-            embed_kernel<float><<<R, 256, 0, s>>>(reinterpret_cast<const float*>(m->embed), tok, d, c.vocab, m->x,
+            embed_kernel<float><<<dim3(R, (d + 255) / 256), 256, 0, s>>>(reinterpret_cast<const float*>(m->embed), tok, d, c.vocab, m->x,
                                                   cap_ptr(0), m->ss, nullptr, nullptr);
         return cudaGetLastError();
     }, "embed"));
@@ -361,7 +354,7 @@ static ks_status forward(ks_model* m, const int32_t* tok, int R, int p0, const u
             GemvArgs g{};
             common(g, m->w_qkv[l], nqkv, d);
             norm_input(g, m->attn_norm[l]);
-            if (bf) { g.wmap = m->map_qkv[l]; g.xmap = m->map_xg[R > 8]; }
+            if (bf) { g.wmap = m->map_qkv[l]; g.xmap = m->map_xg[R - 1]; }
             g.out = m->qkv;
             g.out_ld = nqkv;
             gemv_plan(g, EPI_STORE);
@@ -374,7 +367,7 @@ static ks_status forward(ks_model* m, const int32_t* tok, int R, int p0, const u
             at.rope = m->rope;
             at.q_norm = c.qk_norm ? m->q_norm[l] : nullptr;
             at.k_norm = c.qk_norm ? m->k_norm[l] : nullptr;
-            at.eps = c.rms_eps; at.chunk = kAttnChunk;
+            at.eps = c.rms_eps;
             at.part = m->attn_part; at.n_chunks_max = m->lay.n_chunks_max;
             at.out = m->attn_out; at.out_ld = c.n_q_heads * hd;
             KS_TRY(launch(m, K_ATTN, [&] { return launch_attention(dt, at, s); }, "attention"));
@@ -382,7 +375,7 @@ static ks_status forward(ks_model* m, const int32_t* tok, int R, int p0, const u
 
             GemvArgs o{};
             common(o, m->w_o[l], d, c.n_q_heads * hd);
-            if (bf) { o.wmap = m->map_o[l]; o.xmap = m->map_attn_out[R > 8]; }
+            if (bf) { o.wmap = m->map_o[l]; o.xmap = m->map_attn_out[R - 1]; }
             o.in = m->attn_out;
             o.in_ld = c.n_q_heads * hd;
             resid_output(o, 2 * l + 1);
@@ -393,7 +386,7 @@ static ks_status forward(ks_model* m, const int32_t* tok, int R, int p0, const u
             GemvArgs gu{};
             common(gu, m->w_gate_up[l], c.d_ff, d);
             norm_input(gu, m->mlp_norm[l]);
-            if (bf) { gu.wmap = m->map_gu[l]; gu.xmap = m->map_xg[R > 8]; }
+            if (bf) { gu.wmap = m->map_gu[l]; gu.xmap = m->map_xg[R - 1]; }
             gu.act = m->act;
             gu.act_ld = c.d_ff;
             gemv_plan(gu, EPI_SWIGLU);
@@ -401,7 +394,7 @@ static ks_status forward(ks_model* m, const int32_t* tok, int R, int p0, const u
 
             GemvArgs dn{};
             common(dn, m->w_down[l], d, c.d_ff);
-            if (bf) { dn.wmap = m->map_down[l]; dn.xmap = m->map_act[R > 8]; }
+            if (bf) { dn.wmap = m->map_down[l]; dn.xmap = m->map_act[R - 1]; }
             dn.in = m->act;
             dn.in_ld = c.d_ff;
             resid_output(dn, 2 * l + 2);
@@ -413,7 +406,7 @@ static ks_status forward(ks_model* m, const int32_t* tok, int R, int p0, const u
         GemvArgs lm{};
         common(lm, m->lm_head, c.vocab, d);
         norm_input(lm, m->final_norm);
-        if (bf) { lm.wmap = m->map_lm; lm.xmap = m->map_xg[R > 8]; }
+        if (bf) { lm.wmap = m->map_lm; lm.xmap = m->map_xg[R - 1]; }
         lm.logits = m->logits;
         lm.logits_ld = c.vocab;
         lm.amax_val = m->amax_val;
@@ -572,10 +565,10 @@ ks_status ks_model_create(const ks_config* cfg, const ks_weights* w, void* works
             ok = ok && make_tma_map(&m->map_down[l], m->w_down[l], d, F, 16);
         }
         ok = ok && make_tma_map(&m->map_lm, m->lm_head, cfg->vocab, d, 16);
-        for (int b = 0; b < 2; ++b) {
-            ok = ok && make_tma_map(&m->map_xg[b], m->xg, R, d, 8u << b);
-            ok = ok && make_tma_map(&m->map_attn_out[b], m->attn_out, R, hqd, 8u << b);
-            ok = ok && make_tma_map(&m->map_act[b], m->act, R, F, 8u << b);
+        for (int b = 0; b < R; ++b) {
+            ok = ok && make_tma_map(&m->map_xg[b], m->xg, R, d, b + 1);
+            ok = ok && make_tma_map(&m->map_attn_out[b], m->attn_out, R, hqd, b + 1);
+            ok = ok && make_tma_map(&m->map_act[b], m->act, R, F, b + 1);
         }
         if (!ok) {
             set_error("ks_model_create: TMA descriptor encoding failed");

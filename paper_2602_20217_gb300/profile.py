@@ -6,6 +6,9 @@ average CUDA-event time of each kernel class.  Sized to keep a profiler's
 capture short: a few GB of device memory, a few hundred kernel launches.
 
   python -m paper_2602_20217_gb300.profile --workload llama8b-4k --layers 2 --prompt 512 --steps 3
+
+The speculative steps run inside an NVTX range named "decode", so a profiler
+can skip the prefill (ncu --nvtx --nvtx-include "decode/").
 """
 from __future__ import annotations
 
@@ -44,8 +47,11 @@ def main():
         for k in range(9):
             ks.ks_kernel_timing(m.h, k, True)
     mask = np.array([0, 1] * sh.n_layers, np.uint8)   # draft: MLP sublayers only
+    torch.cuda.synchronize()
+    torch.cuda.nvtx.range_push("decode")              # profilers can filter on this range
     out, st, acc = m.generate(1 << 20, args.gamma, mask=mask, max_steps=args.steps)
     torch.cuda.synchronize()
+    torch.cuda.nvtx.range_pop()
     res = {"workload": wl.name, "layers": sh.n_layers, "prompt": args.prompt, "steps": int(st.steps),
            "accepted": int(st.accepted)}
     if args.timing:
