@@ -203,6 +203,29 @@ ks_status ks_select_mask(const ks_latency* lat, const float* sims, int64_t conte
                          double* objective_out, int32_t* weights_out, void* scratch,
                          size_t scratch_bytes, void* stream);
 
+/* Allocation-free variant of ks_select_mask (the paper has no counterpart:
+ * this is a deployment convenience).  Some callers cannot give this library
+ * any device memory beyond their own inputs and outputs - for example a
+ * plugin inside a host framework that owns every allocation, or a serving
+ * loop that must not call cudaMalloc after start-up because cudaMalloc can
+ * synchronise the device.  For them the knapsack's work tables live in one
+ * array built into the library: a file-scope __device__ buffer of about
+ * 1.1 MB on every GPU that loads the library, held until the process exits.
+ * Same inputs, outputs and results as ks_select_mask, without the scratch
+ * arguments; budget_units must be 0..KS_SELECT_STATIC_MAX_BUDGET (larger
+ * budgets return KS_ERR_INVALID_ARG).  The call allocates nothing: no
+ * cudaMalloc, cudaFree or allocating library routine.
+ * The first call on a device looks up the array's device address
+ * (cudaGetSymbolAddress) with that device current; make that first call
+ * before any stream capture.  All calls share the one array and the kernel
+ * rewrites every table entry it reads, so no state leaks from one call to
+ * the next; two calls whose kernels overlap on the GPU (different streams)
+ * race on the array and must be ordered by the caller. */
+#define KS_SELECT_STATIC_MAX_BUDGET 4095
+ks_status ks_select_mask_static(const ks_latency* lat, const float* sims, int64_t context_len,
+                                int32_t n_sublayers, int32_t budget_units, uint8_t* mask_out,
+                                double* objective_out, int32_t* weights_out, void* stream);
+
 /* ------------------------------------------------- full speculative loop */
 
 typedef struct {

@@ -15,6 +15,7 @@
 #include "internal.h"
 
 #include <cmath>
+#include <mutex>
 
 namespace ks {
 
@@ -201,10 +202,94 @@ cudaError_t launch_select(const ks_latency* lat, const float* sims, int64_t n, i
     return cudaGetLastError();
 }
 
+static ks_status check_latency(const ks_latency* lat, int32_t n) {
+    if (!lat) return KS_ERR_INVALID_ARG;
+    if (lat->kind == 0) {
+        if (!(lat->c1 > 0.0) || !(lat->c2 >= 0.0) || !(lat->c3 >= 0.0) || !std::isfinite(lat->c1) ||
+            !std::isfinite(lat->c2) || !std::isfinite(lat->c3))
+            return KS_ERR_INVALID_ARG;
+        return KS_OK;
+    }
+    if (lat->kind == 1) {
+        if (!lat->units) return KS_ERR_INVALID_ARG;
+        for (int i = 0; i < n; ++i)
+            if (lat->units[i] < 1 || lat->units[i] > 65535) return KS_ERR_INVALID_ARG;
+        return KS_OK;
+    }
+    return KS_ERR_INVALID_ARG;
+}
+
+// ------------------------------------------------ allocation-free variant
+// Work tables of ks_select_mask_static: one array for the whole process on
+// every device that loads the library, sized for KS_SELECT_STATIC_MAX_BUDGET
+// units and kMaxItems sublayers (about 1.1 MB).  Host code may not use the
+// symbol as an address; the device address comes from cudaGetSymbolAddress.
+constexpr int kStaticCap = KS_SELECT_STATIC_MAX_BUDGET;
+constexpr size_t kStaticScratchBytes =
+    ((sizeof(long long) * 2 * ((size_t)kStaticCap + 1) + (size_t)kMaxItems * ((size_t)kStaticCap + 1)) + 255) / 256 *
+    256;
+static __device__ __align__(256) unsigned char g_select_scratch[kStaticScratchBytes];
+
+static std::mutex g_static_mu;
+static void* g_static_ptr[128] = {};
+
+// Device address of g_select_scratch on the current device, looked up once
+// per device (the first call on a device does the lookup).
+static cudaError_t static_scratch(void** out) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 128) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lock(g_static_mu);
+    if (g_static_ptr[dev] == nullptr) {
+        void* p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_select_scratch);
+        if (e != cudaSuccess) return e;
+        g_static_ptr[dev] = p;
+    }
+    *out = g_static_ptr[dev];
+    return cudaSuccess;
+}
+
 }  // namespace ks
 
 // ------------------------------------------------------------------- C ABI
 using namespace ks;
+
+extern "C" ks_status ks_select_mask_static(const ks_latency* lat, const float* sims, int64_t context_len,
+                                           int32_t n_sublayers, int32_t budget_units, uint8_t* mask_out,
+                                           double* objective_out, int32_t* weights_out, void* stream) {
+    if (!sims || !mask_out) {
+        set_error("ks_select_mask_static: null pointer");
+        return KS_ERR_INVALID_ARG;
+    }
+    if (n_sublayers < 2 || n_sublayers > kMaxItems || (n_sublayers & 1) || context_len < 0) {
+        set_error("ks_select_mask_static: bad n_sublayers / context_len");
+        return KS_ERR_INVALID_ARG;
+    }
+    if (budget_units < 0 || budget_units > kStaticCap) {
+        set_error("ks_select_mask_static: budget_units %d outside 0..%d (the size of the built-in tables)",
+                  budget_units, kStaticCap);
+        return KS_ERR_INVALID_ARG;
+    }
+    if (check_latency(lat, n_sublayers) != KS_OK) {
+        set_error("ks_select_mask_static: bad latency model");
+        return KS_ERR_INVALID_ARG;
+    }
+    void* scratch = nullptr;
+    cudaError_t e = static_scratch(&scratch);
+    if (e != cudaSuccess) {
+        set_error("ks_select_mask_static: cudaGetSymbolAddress: %s", cudaGetErrorString(e));
+        return KS_ERR_CUDA;
+    }
+    e = launch_select(lat, sims, context_len, n_sublayers, budget_units, -1.0, mask_out, objective_out, weights_out,
+                      nullptr, scratch, budget_units, reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) {
+        set_error("ks_select_mask_static: %s", cudaGetErrorString(e));
+        return KS_ERR_CUDA;
+    }
+    return KS_OK;
+}
 
 extern "C" ks_status ks_cosine(const void* X, const void* Y, int32_t dtype, int64_t n_pairs, int32_t rows,
                                int32_t d, int64_t pair_stride, const int32_t* row_index, float* out,
@@ -232,22 +317,6 @@ extern "C" size_t ks_select_scratch_bytes(int32_t n_sublayers, int32_t budget_un
     return select_scratch_bytes(n_sublayers, budget_units);
 }
 
-static ks_status check_latency(const ks_latency* lat, int32_t n) {
-    if (!lat) return KS_ERR_INVALID_ARG;
-    if (lat->kind == 0) {
-        if (!(lat->c1 > 0.0) || !(lat->c2 >= 0.0) || !(lat->c3 >= 0.0) || !std::isfinite(lat->c1) ||
-            !std::isfinite(lat->c2) || !std::isfinite(lat->c3))
-            return KS_ERR_INVALID_ARG;
-        return KS_OK;
-    }
-    if (lat->kind == 1) {
-        if (!lat->units) return KS_ERR_INVALID_ARG;
-        for (int i = 0; i < n; ++i)
-            if (lat->units[i] < 1 || lat->units[i] > 65535) return KS_ERR_INVALID_ARG;
-        return KS_OK;
-    }
-    return KS_ERR_INVALID_ARG;
-}
 
 extern "C" ks_status ks_select_mask(const ks_latency* lat, const float* sims, int64_t context_len,
                                     int32_t n_sublayers, int32_t budget_units, uint8_t* mask_out,

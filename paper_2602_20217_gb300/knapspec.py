@@ -80,6 +80,8 @@ _SIGS = {
     "ks_select_scratch_bytes": (C.c_size_t, [C.c_int32, C.c_int32]),
     "ks_select_mask": (C.c_int, [C.POINTER(KsLatency), C.c_void_p, C.c_int64, C.c_int32, C.c_int32, C.c_void_p,
                                  C.c_void_p, C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p]),
+    "ks_select_mask_static": (C.c_int, [C.POINTER(KsLatency), C.c_void_p, C.c_int64, C.c_int32, C.c_int32,
+                                        C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]),
     "ks_generate_speculative": (C.c_int, [C.c_void_p, C.POINTER(KsSpecParams), C.c_int32, C.c_void_p,
                                           C.POINTER(KsSpecStats), C.c_void_p]),
     "ks_debug_read": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32, C.c_int32, C.c_int32, C.c_void_p, C.c_size_t]),
@@ -248,6 +250,17 @@ def ks_select_mask(lat: KsLatency, sims, context_len: int, n_sublayers: int, bud
     check(load().ks_select_mask(C.byref(lat), _ptr(sims), context_len, n_sublayers, budget_units,
                                 _ptr(mask_out), _ptr(objective_out), _ptr(weights_out), _ptr(scratch),
                                 scratch_bytes, _stream_ptr(stream)), "ks_select_mask")
+
+
+KS_SELECT_STATIC_MAX_BUDGET = 4095
+
+
+def ks_select_mask_static(lat: KsLatency, sims, context_len: int, n_sublayers: int, budget_units: int, mask_out,
+                          objective_out, weights_out, stream=None):
+    """ks_select_mask with the library's built-in work tables (no scratch argument)."""
+    check(load().ks_select_mask_static(C.byref(lat), _ptr(sims), context_len, n_sublayers, budget_units,
+                                       _ptr(mask_out), _ptr(objective_out), _ptr(weights_out),
+                                       _stream_ptr(stream)), "ks_select_mask_static")
 
 
 def ks_generate_speculative(h: int, params: KsSpecParams, n_tokens: int):
