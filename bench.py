@@ -34,6 +34,22 @@ UNIT = "tokens/s"
 DEFAULT_WORKLOAD = "llama8b-4k"
 
 
+def gateup_traffic():
+    """DRAM bytes (read + write) of one gate/up launch from the committed ncu
+    capture, or None when the kernel's sources changed since the capture."""
+    import hashlib
+    try:
+        with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
+            rec = json.load(f)["gemv_stream_kernel<1, 2>"]
+        h = hashlib.sha256()
+        for name in rec["source_files"]:
+            with open(os.path.join(ROOT, name), "rb") as f:
+                h.update(f.read())
+        return float(rec["traffic_bytes_per_launch"]) if h.hexdigest() == rec["source_sha256"] else None
+    except Exception:
+        return None
+
+
 def peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -230,10 +246,12 @@ def gpu_arm(args):
                 if os.path.isdir(os.path.join(ROOT, "gpurun_out")) else f"/tmp/ks_clocks_{rank}.csv")
     clocks = ClockSampler(clk_path)
     with clocks:
+        torch.cuda.nvtx.range_push("timed")  # lets a profiler capture exactly these steps
         ev0.record(stream)
         _, st, acc = ks.ks_generate_speculative(h, params(args.steps), 1 << 30)
         ev1.record(stream)
         torch.cuda.synchronize()
+        torch.cuda.nvtx.range_pop()
     if dist:
         dist.barrier()
     ms = ev0.elapsed_time(ev1)
@@ -295,8 +313,9 @@ def gpu_arm(args):
                     "d2h_bytes_per_step": (d2h1 - d2h0) / max(1, est.steps)},
             "gpu_launches": launches,
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                         "frac": achieved / peak, "traffic": None,
-                         "kernel": "gemv_kernel SwiGLU (gate/up)", "peak_source": peak_kind,
+                         "frac": achieved / peak,
+                         "traffic": gateup_traffic() if wl.name == "llama8b-4k" else None,
+                         "kernel": "gemv_stream_kernel<1, 2> (SwiGLU gate/up)", "peak_source": peak_kind,
                          "launches_timed": gu_n, "bytes_per_launch": gu_bytes},
             "kernels_us": {k: round(1e3 * v[1] / max(1, v[0]), 2) for k, v in kt.items()},
             "clocks": clocks.summary(local),
