@@ -178,6 +178,18 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(rows)}
 
 
+def reduce_over_ranks(ms: float, tokens: float, dist=None, device="cpu"):
+    """Replicas: the job's time is the slowest rank's, its tokens the sum
+    over ranks.  Returns (max ms, total tokens)."""
+    import torch
+    a = torch.tensor([float(ms)], dtype=torch.float64, device=device)
+    b = torch.tensor([float(tokens)], dtype=torch.float64, device=device)
+    if dist is not None:
+        dist.all_reduce(a, op=dist.ReduceOp.MAX)
+        dist.all_reduce(b, op=dist.ReduceOp.SUM)
+    return float(a[0]), float(b[0])
+
+
 def gpu_arm(args):
     import torch
     rank = int(os.environ.get("RANK", "0"))
@@ -209,6 +221,10 @@ def gpu_arm(args):
         torch.cuda.synchronize()
         return time.time() - t
 
+    def rewind():   # back to the post-prefill state; the prompt's KV cache is reused
+        model.rewind()
+        torch.cuda.synchronize()
+
     # Latency model of App. C measured on this GPU at the prompt's context:
     # c1 = MLP sublayer (gate/up + down), c3 = the Attn sublayer's
     # context-independent kernels (QKV, merge, O-proj), c2 = attention-kernel
@@ -231,10 +247,10 @@ def gpu_arm(args):
                                int(max_steps))
 
     # warm-up
-    prefill()
+    rewind()
     ks.ks_generate_speculative(h, params(args.warmup), 1 << 30)
     # timed region: exactly K speculation steps, device time on the model's stream
-    prefill()
+    rewind()
     ks.ks_kernel_timing(h, ks.KLASS["gateup"], True)
     launches0 = ks.ks_launch_count(h)
     if dist:
@@ -262,7 +278,7 @@ def gpu_arm(args):
 
     # e2e: the public call with host output buffers, wall clock, for a
     # generation job of e2e_tokens tokens (the prompt already prefilled)
-    prefill()
+    rewind()
     h2d0, d2h0 = ks.ks_transfer_bytes(h)
     t0 = time.perf_counter()
     out, est, eacc = ks.ks_generate_speculative(h, params(0), args.e2e_tokens)
@@ -270,20 +286,39 @@ def gpu_arm(args):
     h2d1, d2h1 = ks.ks_transfer_bytes(h)
     e2e_tok = int(est.steps + est.accepted)
     # the same library's plain greedy decode of the same job
-    prefill()
+    rewind()
     t0 = time.perf_counter()
     ar = ks.ks_decode_greedy(h, args.e2e_tokens)
     ar_s = time.perf_counter() - t0
     lossless = bool(np.array_equal(out, ar))
 
-    vals = torch.tensor([ms, float(tokens)], dtype=torch.float64, device="cuda")
-    if dist:
-        a = vals[0:1].clone()
-        b = vals[1:2].clone()
-        dist.all_reduce(a, op=dist.ReduceOp.MAX)
-        dist.all_reduce(b, op=dist.ReduceOp.SUM)
-        vals = torch.cat([a, b])
-    ms_max, tok_all = float(vals[0]), float(vals[1])
+    sweep = []
+    if args.sweep:
+        # accepted tokens/s (device time) of e2e_tokens-token jobs over a grid
+        # of knapsack budgets and draft lengths, next to the greedy decode
+        def timed(fn):
+            rewind()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            r = fn()
+            e1.record(stream)
+            torch.cuda.synchronize()
+            return r, e0.elapsed_time(e1) * 1e-3
+        _, t_ar = timed(lambda: ks.ks_decode_greedy(h, args.e2e_tokens))
+        sweep.append({"policy": "greedy", "tokens_per_s": (args.e2e_tokens - 1) / t_ar})
+        for g in sorted({int(x) for x in args.sweep_gammas.split(",")}):
+            for bf in [float(x) for x in args.sweep_budgets.split(",")]:
+                p = ks.KsSpecParams(g, 1, None, lat, bf, int(args.resolve_every), 0)
+                (o, sst, _a), t = timed(lambda: ks.ks_generate_speculative(h, p, args.e2e_tokens))
+                n_tok = int(sst.steps + sst.accepted)
+                sweep.append({"gamma": g, "budget_frac": bf, "tokens_per_s": n_tok / t,
+                              "vs_greedy": (n_tok / t) / ((args.e2e_tokens - 1) / t_ar),
+                              "alpha": float(sst.accepted) / max(1, sst.drafted),
+                              "tokens_per_step": n_tok / max(1, sst.steps),
+                              "skipped_attn_mlp": [int(sst.attn_skipped), int(sst.mlp_skipped)]})
+
+    ms_max, tok_all = reduce_over_ranks(ms, tokens, dist, "cuda")
 
     if rank == 0:
         peak, peak_kind = peaks()
@@ -320,6 +355,8 @@ def gpu_arm(args):
             "kernels_us": {k: round(1e3 * v[1] / max(1, v[0]), 2) for k, v in kt.items()},
             "clocks": clocks.summary(local),
         }
+        if sweep:
+            line["sweep_device_time"] = sweep
         if not args.no_cpu_baseline and world == 1:
             try:
                 line["cpu_baseline"] = cpu_baseline(wl.name)
@@ -343,6 +380,10 @@ def main():
     ap.add_argument("--resolve-every", dest="resolve_every", type=int, default=1)
     ap.add_argument("--e2e-tokens", dest="e2e_tokens", type=int, default=256)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--sweep", action="store_true",
+                    help="also time jobs over a grid of knapsack budgets and draft lengths")
+    ap.add_argument("--sweep-budgets", dest="sweep_budgets", default="0.4,0.5,0.6,0.7,0.8")
+    ap.add_argument("--sweep-gammas", dest="sweep_gammas", default="2,4,6")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

@@ -28,8 +28,10 @@
  *  - Every call returns a ks_status and never aborts, traps or exits.
  *    Invalid arguments are rejected before any work is enqueued.  CUDA errors
  *    are reported as KS_ERR_CUDA (the message is kept per thread, see
- *    ks_last_error).  No kernel spins on a flag; no call waits without a
- *    bound other than a stream synchronisation.
+ *    ks_last_error).  No kernel waits on another launch; the pipeline waits
+ *    inside a kernel (TMA barriers) give up after 2 s, record the fact in a
+ *    device status word and return, and the next synchronising call reports
+ *    KS_ERR_TIMEOUT.
  *  - One handle is used by one host thread at a time and issues all work on
  *    the stream given at creation.
  *  - Greedy argmax ties resolve to the lowest token id.
@@ -50,7 +52,7 @@ typedef enum {
     KS_ERR_CUDA = 2,          /* a CUDA runtime call or kernel launch failed        */
     KS_ERR_WORKSPACE = 3,     /* the workspace is smaller than required             */
     KS_ERR_CAPACITY = 4,      /* KV capacity (max_seq) or row capacity exceeded     */
-    KS_ERR_TIMEOUT = 5,       /* reserved: a bounded device wait gave up            */
+    KS_ERR_TIMEOUT = 5,       /* a bounded device-side wait gave up (2 s limit)     */
     KS_ERR_UNSUPPORTED = 6,   /* shape/dtype outside what the kernels implement     */
     KS_ERR_STATE = 7          /* call out of order (e.g. draft before prefill)      */
 } ks_status;
@@ -132,6 +134,14 @@ ks_status ks_model_destroy(ks_model* m);
  * last hist_init_rows prompt rows, and set the pending token to the greedy
  * next token, written to *next_token (host).  Resets any previous sequence. */
 ks_status ks_prefill(ks_model* m, const int32_t* tokens, int32_t n, int32_t* next_token);
+
+/* Return to the state right after the last ks_prefill without recomputing the
+ * prompt: decoding writes K/V only at positions at or past the prompt length,
+ * so the prompt's cache is still valid; the committed length, the pending
+ * token (also written to *next_token, host) and the history are restored.
+ * Serves several generations from one long prompt.  (An addition of this
+ * library; the paper has no counterpart.)  KS_ERR_STATE before any prefill. */
+ks_status ks_rewind(ks_model* m, int32_t* next_token);
 
 /* a1 (Sec. 2, Sec. 2.2): gamma (1 <= gamma < max_rows) greedy draft tokens
  * from f^(S), S = { i : mask[i-1] != 0 } (host uint8[2L]; odd 1-based

@@ -86,7 +86,7 @@ static size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
 struct Layout {
     size_t kv, rope, x, ss, xg, qkv, attn_out, act, attn_part, gemv_part, counters, logits, amax_val,
-        amax_idx, tok, hist, hist_idx, sims, mask, obj, wts, select, total;
+        amax_idx, tok, hist, hist_snap, hist_idx, sims, mask, obj, wts, select, total;
     int n_chunks_max;
     size_t gemv_part_floats;
     int counters_n;
@@ -154,6 +154,7 @@ static Layout make_layout(const ks_config* c) {
     // tokens: rows[R+1] | target[R] | result[R+3] | err | prompt/out[max_seq]
     L.tok = take(sizeof(int) * ((size_t)3 * R + 8 + c->max_seq));
     L.hist = take(sizeof(float) * (size_t)(nsub + 1) * L.hist_slots * R * d);
+    L.hist_snap = take(sizeof(float) * (size_t)(nsub + 1) * R * d);  // the prefill's history entry
     L.hist_idx = take(sizeof(int) * (size_t)L.hist_slots * R);
     L.sims = take(sizeof(float) * nsub);
     L.mask = take(nsub);
@@ -189,7 +190,7 @@ struct ks_model {
     Layout lay;
     // carved pointers
     char* kv;
-    float *rope, *x, *ss, *qkv, *attn_part, *gemv_part, *logits, *amax_val, *hist, *sims;
+    float *rope, *x, *ss, *qkv, *attn_part, *gemv_part, *logits, *amax_val, *hist, *hist_snap, *sims;
     __nv_bfloat16* xg;
     void *attn_out, *act, *select;
     int *counters, *amax_idx, *rows, *target, *result, *err, *seq, *hist_idx;
@@ -203,6 +204,9 @@ struct ks_model {
     bool have_seq = false;
     int p = 0;
     int pending = 0;
+    int prompt_len = 0;       // state right after the last prefill, for ks_rewind
+    int prompt_pending = 0;
+    int prompt_rows = 0;
     int last_gamma = -1;
     int last_pass_rows = 0;
     std::vector<int> slot_off, slot_cnt;  // history ring rows per slot
@@ -542,6 +546,7 @@ ks_status ks_model_create(const ks_config* cfg, const ks_weights* w, void* works
     m->err = tok + (3 * R + 4);
     m->seq = tok + (3 * R + 8);
     m->hist = reinterpret_cast<float*>(b + lay.hist);
+    m->hist_snap = reinterpret_cast<float*>(b + lay.hist_snap);
     m->hist_idx = reinterpret_cast<int*>(b + lay.hist_idx);
     m->sims = reinterpret_cast<float*>(b + lay.sims);
     m->mask_dev = reinterpret_cast<uint8_t*>(b + lay.mask);
@@ -627,6 +632,17 @@ ks_status ks_model_destroy(ks_model* m) {
     return KS_OK;
 }
 
+// The history after a prefill: one entry holding the last hist_init_rows of
+// the prompt's final chunk (lastlen rows captured in slot 0).
+static void reset_history(ks_model* m, int lastlen) {
+    m->last_gamma = -1;
+    std::fill(m->slot_cnt.begin(), m->slot_cnt.end(), 0);
+    const int init = std::min(m->cfg.hist_init_rows, lastlen);
+    m->slot_off[0] = lastlen - init;
+    m->slot_cnt[0] = init;
+    m->hist_next = 1;
+}
+
 ks_status ks_prefill(ks_model* m, const int32_t* tokens, int32_t n, int32_t* next_token) {
     if (!m || !tokens || !next_token) {
         set_error("ks_prefill: null argument");
@@ -647,6 +663,7 @@ ks_status ks_prefill(ks_model* m, const int32_t* tokens, int32_t n, int32_t* nex
             return KS_ERR_INVALID_ARG;
         }
     m->have_seq = false;
+    m->prompt_len = 0;
     std::memcpy(m->h_buf, tokens, sizeof(int32_t) * n);
     KS_CUDA(cudaMemcpyAsync(m->seq, m->h_buf, sizeof(int32_t) * n, cudaMemcpyHostToDevice, m->stream), "prompt upload");
     m->h2d += sizeof(int32_t) * n;
@@ -673,12 +690,44 @@ ks_status ks_prefill(ks_model* m, const int32_t* tokens, int32_t n, int32_t* nex
     *next_token = m->pending;
     m->p = n;
     m->have_seq = true;
-    m->last_gamma = -1;
-    std::fill(m->slot_cnt.begin(), m->slot_cnt.end(), 0);
-    const int init = std::min(c.hist_init_rows, lastlen);
-    m->slot_off[init_slot] = lastlen - init;
-    m->slot_cnt[init_slot] = init;
-    m->hist_next = 1;
+    m->prompt_len = n;
+    m->prompt_pending = m->pending;
+    m->prompt_rows = lastlen;
+    // keep the prefill's history entry (slot 0 of every plane) for ks_rewind
+    const size_t row_bytes = sizeof(float) * (size_t)c.max_rows * c.d_model;
+    KS_CUDA(cudaMemcpy2DAsync(m->hist_snap, row_bytes, m->hist, row_bytes * m->lay.hist_slots, row_bytes,
+                              m->nsub + 1, cudaMemcpyDeviceToDevice, m->stream),
+            "history snapshot");
+    reset_history(m, lastlen);
+    return KS_OK;
+}
+
+ks_status ks_rewind(ks_model* m, int32_t* next_token) {
+    if (!m || !next_token) {
+        set_error("ks_rewind: null argument");
+        return KS_ERR_INVALID_ARG;
+    }
+    if (m->prompt_len < 1) {
+        set_error("ks_rewind: no prompt (call ks_prefill first)");
+        return KS_ERR_STATE;
+    }
+    // Decode steps write K/V only at positions >= the prompt length, so the
+    // prompt's cache is intact; restore the pending token and the history.
+    const ks_config& c = m->cfg;
+    m->have_seq = false;
+    m->h_buf[0] = m->prompt_pending;
+    KS_CUDA(cudaMemcpyAsync(m->rows, m->h_buf, sizeof(int32_t), cudaMemcpyHostToDevice, m->stream), "pending");
+    m->h2d += sizeof(int32_t);
+    const size_t row_bytes = sizeof(float) * (size_t)c.max_rows * c.d_model;
+    KS_CUDA(cudaMemcpy2DAsync(m->hist, row_bytes * m->lay.hist_slots, m->hist_snap, row_bytes, row_bytes,
+                              m->nsub + 1, cudaMemcpyDeviceToDevice, m->stream),
+            "history restore");
+    KS_TRY(sync(m, "ks_rewind"));
+    m->p = m->prompt_len;
+    m->pending = m->prompt_pending;
+    m->have_seq = true;
+    reset_history(m, m->prompt_rows);
+    *next_token = m->pending;
     return KS_OK;
 }
 

@@ -69,6 +69,7 @@ _SIGS = {
                                   C.c_void_p, C.POINTER(C.c_void_p)]),
     "ks_model_destroy": (C.c_int, [C.c_void_p]),
     "ks_prefill": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.POINTER(C.c_int32)]),
+    "ks_rewind": (C.c_int, [C.c_void_p, C.POINTER(C.c_int32)]),
     "ks_draft": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p]),
     "ks_verify": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.POINTER(C.c_int32), C.c_void_p,
                             C.POINTER(C.c_int32)]),
@@ -189,6 +190,12 @@ def ks_prefill(h: int, tokens) -> int:
     t = np.ascontiguousarray(tokens, dtype=np.int32)
     nxt = C.c_int32()
     check(load().ks_prefill(h, t.ctypes.data, len(t), C.byref(nxt)), "ks_prefill")
+    return nxt.value
+
+
+def ks_rewind(h: int) -> int:
+    nxt = C.c_int32()
+    check(load().ks_rewind(h, C.byref(nxt)), "ks_rewind")
     return nxt.value
 
 

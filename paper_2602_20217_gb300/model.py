@@ -32,6 +32,9 @@ class Model:
     def prefill(self, tokens) -> int:
         return ks.ks_prefill(self.h, tokens)
 
+    def rewind(self) -> int:
+        return ks.ks_rewind(self.h)
+
     def draft(self, mask, gamma: int):
         return ks.ks_draft(self.h, mask, gamma)
 

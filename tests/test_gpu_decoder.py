@@ -240,3 +240,34 @@ def test_capacity_and_state_errors():
         m.prefill(np.array([5, 2000], np.int32))
     assert e.value.status == ks.KS_ERR_INVALID_ARG
     m.close()
+
+
+def test_rewind_reuses_the_prompt():
+    """ks_rewind restores the post-prefill state: the generations that follow
+    are bit-identical to ones after a fresh prefill (history included)."""
+    from paper_2602_20217_gb300 import knapspec as ks
+    from paper_2602_20217_gb300 import synth
+    shape = small_bf16(128, True)
+    prompt = synth.prompt_tokens(shape, 300, seed=1)
+    m = make(shape, 512)
+    with pytest.raises(ks.KsError) as e:
+        m.rewind()
+    assert e.value.status == ks.KS_ERR_STATE
+    pend = m.prefill(prompt)
+    hist0, sims0 = m.history(), m.history_similarities()[0]
+    ar = m.decode_greedy(24)
+    units = synth.unit_table(shape.n_sublayers, seed=2)
+    lat = ks.latency(1, units=units)
+    assert m.prefill(prompt) == pend
+    spec = m.generate(40, 4, latency=lat, budget_frac=0.6, resolve_every=1)
+    assert list(spec[0][:24]) == list(ar)
+    for _ in range(2):
+        assert m.rewind() == pend
+        assert m.position() == (300, pend)
+        assert np.array_equal(m.history(), hist0)
+        assert np.array_equal(m.history_similarities()[0], sims0)
+        assert list(m.decode_greedy(24)) == list(ar)
+        m.rewind()
+        out, st, acc = m.generate(40, 4, latency=lat, budget_frac=0.6, resolve_every=1)
+        assert list(out) == list(spec[0]) and np.array_equal(acc, spec[2])
+    m.close()
