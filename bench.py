@@ -34,18 +34,21 @@ UNIT = "tokens/s"
 DEFAULT_WORKLOAD = "llama8b-4k"
 
 
-def gateup_traffic():
-    """DRAM bytes (read + write) of one gate/up launch from the committed ncu
-    capture, or None when the kernel's sources changed since the capture."""
+def chain_traffic(bytes_per_launch: float):
+    """DRAM bytes (read + write) per chain launch, scaled from the committed ncu
+    capture (traffic per algorithmic byte x this run's algorithmic bytes per
+    launch), or None when the kernel's sources changed since the capture."""
     import hashlib
     try:
         with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
-            rec = json.load(f)["gemv_stream_kernel<1, 2>"]
+            rec = json.load(f)["chain_kernel"]
         h = hashlib.sha256()
         for name in rec["source_files"]:
             with open(os.path.join(ROOT, name), "rb") as f:
                 h.update(f.read())
-        return float(rec["traffic_bytes_per_launch"]) if h.hexdigest() == rec["source_sha256"] else None
+        if h.hexdigest() != rec["source_sha256"]:
+            return None
+        return float(rec["traffic_per_algorithmic_byte"]) * bytes_per_launch
     except Exception:
         return None
 
@@ -230,11 +233,12 @@ def gpu_arm(args):
     # context-independent kernels (QKV, merge, O-proj), c2 = attention-kernel
     # time / context length.
     t_prefill = prefill()
-    for k in range(9):
+    split = [k for name, k in ks.KLASS.items() if name != "chain"]   # one projection per launch
+    for k in split:
         ks.ks_kernel_timing(h, k, True)
     model.decode_greedy(8)
-    kt = {name: ks.ks_kernel_time(h, k) for name, k in ks.KLASS.items()}
-    for k in range(9):
+    kt = {name: ks.ks_kernel_time(h, k) for name, k in ks.KLASS.items() if name != "chain"}
+    for k in split:
         ks.ks_kernel_timing(h, k, False)
     per = lambda name: kt[name][1] / max(1, kt[name][0])
     c1 = per("gateup") + per("down")
@@ -251,7 +255,7 @@ def gpu_arm(args):
     ks.ks_generate_speculative(h, params(args.warmup), 1 << 30)
     # timed region: exactly K speculation steps, device time on the model's stream
     rewind()
-    ks.ks_kernel_timing(h, ks.KLASS["gateup"], True)
+    ks.ks_kernel_timing(h, ks.KLASS["chain"], True)
     launches0 = ks.ks_launch_count(h)
     if dist:
         dist.barrier()
@@ -272,8 +276,9 @@ def gpu_arm(args):
         dist.barrier()
     ms = ev0.elapsed_time(ev1)
     launches = ks.ks_launch_count(h) - launches0
-    gu_n, gu_ms = ks.ks_kernel_time(h, ks.KLASS["gateup"])
-    ks.ks_kernel_timing(h, ks.KLASS["gateup"], False)
+    ch_n, ch_ms = ks.ks_kernel_time(h, ks.KLASS["chain"])
+    ch_bytes = ks.ks_kernel_bytes(h, ks.KLASS["chain"])
+    ks.ks_kernel_timing(h, ks.KLASS["chain"], False)
     tokens = int(st.steps + st.accepted)
 
     # e2e: the public call with host output buffers, wall clock, for a
@@ -322,9 +327,9 @@ def gpu_arm(args):
 
     if rank == 0:
         peak, peak_kind = peaks()
-        gu_bytes = 2 * sh.d_ff * sh.d_model * sh.elem_bytes   # weight bytes one gate/up launch must read
-        gu_avg_ms = gu_ms / max(1, gu_n)
-        achieved = gu_bytes / (gu_avg_ms * 1e-3) / 1e9
+        # dominant kernel: the chained projections; algorithmic bytes = the
+        # weight bytes of the projections each launch ran
+        achieved = ch_bytes / (ch_ms * 1e-3) / 1e9 if ch_ms > 0 else 0.0
         line = {
             "metric": METRIC, "value": tok_all / (ms_max * 1e-3), "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_max / args.steps,
@@ -349,9 +354,10 @@ def gpu_arm(args):
             "gpu_launches": launches,
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak,
-                         "traffic": gateup_traffic() if wl.name == "llama8b-4k" else None,
-                         "kernel": "gemv_stream_kernel<1, 2> (SwiGLU gate/up)", "peak_source": peak_kind,
-                         "launches_timed": gu_n, "bytes_per_launch": gu_bytes},
+                         "traffic": chain_traffic(ch_bytes / max(1, ch_n)) if wl.name == "llama8b-4k" else None,
+                         "kernel": "chain_kernel (chained projections)", "peak_source": peak_kind,
+                         "launches_timed": ch_n, "bytes_per_launch": ch_bytes / max(1, ch_n),
+                         "time_share": ch_ms / ms},
             "kernels_us": {k: round(1e3 * v[1] / max(1, v[0]), 2) for k, v in kt.items()},
             "clocks": clocks.summary(local),
         }

@@ -281,11 +281,17 @@ ks_status ks_debug_read(ks_model* m, int32_t what, int32_t layer, int32_t start,
 
 /* Per-kernel timing with CUDA events on the model's stream.  While enabled,
  * every launch of the kernel class `klass` (0 QKV, 1 attention, 2 merge,
- * 3 O-proj, 4 gate/up, 5 down, 6 LM head, 7 embed, 8 accept) is bracketed
- * by events; ks_kernel_time returns the launches and total milliseconds
- * since enabling.  Enabling resets the counters. */
+ * 3 O-proj, 4 gate/up, 5 down, 6 LM head, 7 embed, 8 accept, 9 chained
+ * projections) is bracketed by events; ks_kernel_time returns the launches
+ * and total milliseconds since enabling.  Enabling resets the counters.
+ * bf16 models run the projections between two attention cores as one chained
+ * launch (class 9); while any of classes 0, 3, 4, 5, 6 is enabled they run
+ * one projection per launch instead, so that each can be timed alone.
+ * ks_kernel_bytes: weight bytes the timed launches of the class had to read
+ * (the algorithmic bytes of the projection classes; 0 for the others). */
 ks_status ks_kernel_timing(ks_model* m, int32_t klass, int32_t enable);
 ks_status ks_kernel_time(ks_model* m, int32_t klass, int64_t* launches, double* total_ms);
+ks_status ks_kernel_bytes(const ks_model* m, int32_t klass, double* bytes);
 
 /* Launch counter: kernels this handle has launched since creation. */
 int64_t ks_launch_count(const ks_model* m);

@@ -1,33 +1,18 @@
-// Skinny GEMM kernels for the decode / verify passes (R <= 16 activation rows).
+// Skinny GEMM kernel for fp32 models (the tiny parity workload), plus the
+// TMA descriptor helper used by the bf16 chain kernel.
 //
-// Y[r][n] = sum_k W[n][k] A[r][k]: the per-token projections of the Attn and
-// MLP sublayers and the LM head (Sec. 2 decoder; every pass of a1 / a2).  At
-// R <= 16 rows the work is a stream over the weights (at most 16 flop per
-// weight byte pair), so the bf16 kernel is built to keep HBM busy:
-//  * persistent and warp-specialised: one CTA per SM; a producer warp claims
-//    work items (16 output features over the full K) and streams their
-//    weight and activation tiles with 2-D TMA into a multi-stage shared
-//    memory ring (about 150-190 KB in flight per SM, no registers held);
-//    four consumer warps split each stage's columns and multiply;
-//  * the tiles are fed as the A operand of mma.sync.m16n8k16 (16 weight rows x
-//    16 k) and the activation rows as B (16 k x 8 rows); the k-slots of A and
-//    B are permuted identically so each lane reads 8 contiguous weights and 8
-//    contiguous activations; column j of the result depends only on
-//    activation row j, so a row computed alone (greedy decode) and the same
-//    row inside a gamma+1-row verify pass are bit-identical;
-//  * the consumer warps' K quarters are added in warp order (bf16), K slices
-//    of the fp32 kernel in slice order by the last CTA of a group (an atomic
-//    ticket, no waiting): results depend only on (N, K), never on R or on
-//    which CTA did what;
-//  * prologue: optional RMSNorm of the fp32 residual, with the row's sum of
-//    squares assembled from per-64-feature partials that the residual's
-//    producer wrote (embed or a residual epilogue), summed in group order;
-//    epilogues: plain store (QKV), residual add with optional history capture
-//    and the new partial sums of squares (W_o, W_down), SwiGLU (gate and up
-//    rows paired in one warp), LM head logits with a per-row argmax (ties to
-//    the lowest id).
-// fp32 models (the tiny parity workload) use a simpler CUDA-core kernel with
-// the same tile ownership, epilogues and split rule.
+// Y[r][n] = sum_k W[n][k] A[r][k] for R <= 16 rows: the per-token
+// projections of the Attn and MLP sublayers and the LM head (Sec. 2 decoder;
+// every pass of a1 / a2).  One CTA per (64-feature group, K slice); each
+// warp computes 16 features with CUDA-core dot products and hands its results
+// over in the mma fragment layout the bf16 path uses, so both share one set
+// of epilogues: plain store (QKV), residual add with optional history capture
+// and partial sums of squares (W_o, W_down), SwiGLU (gate and up rows paired
+// in one warp), LM head logits with a per-row argmax (ties to the lowest id).
+// K slices are added in slice order by the last CTA of a group (an atomic
+// ticket, no waiting): results depend only on (N, K), never on R.  The
+// optional RMSNorm prologue builds each row's sum of squares from the
+// per-16-feature partials that the residual's producer wrote, in group order.
 #include "common.cuh"
 #include "internal.h"
 
@@ -40,9 +25,6 @@ namespace ks {
 constexpr int kGemvWarps = 4;
 constexpr int kRowsPerCta = 16 * kGemvWarps;  // output features per group (CTA or work item)
 constexpr int kMaxRows = 16;
-constexpr int kKT = 128;                      // k columns per streamed weight tile
-constexpr int kKP = kKT + 32;                 // tile row pitch (elements): conflict-free LDS.128
-constexpr int kMaxKc = 1024;                  // largest K slice of a bf16 work item
 // counters: [0] next work item, [1] finished CTAs, [2 + g] ticket of group g
 
 __host__ __device__ __forceinline__ int div_up(int a, int b) { return (a + b - 1) / b; }
@@ -50,7 +32,7 @@ __host__ __device__ __forceinline__ int div_up(int a, int b) { return (a + b - 1
 int gemv_grid_x(int N) { return div_up(N, kRowsPerCta); }
 int gemv_groups(int N, int dtype) { return dtype == 1 ? div_up(N, 16) : div_up(N, kRowsPerCta); }
 
-static int sm_count() {
+int sm_count() {
     static int n = 0;
     if (n == 0) {
         int dev = 0;
@@ -383,380 +365,8 @@ __global__ void __launch_bounds__(128) gemv_f32_kernel(const GemvArgs a) {
     }
 }
 
-// ------------------------------------------------- bf16 streaming kernel
-// Work item = 16 output features (16 weight rows, or 16 gate + 16 up rows)
-// over the full K.  A ring stage holds NB x 256 columns of the item's weight
-// rows (one 256 x 16 TMA box per 256 columns and row block) and of its R
-// activation rows (256 x R boxes), rows 512 bytes apart.  The four
-// consumer warps split each stage's columns evenly; at the end of an item
-// their partial fragments are added in warp order in shared memory.
-//
-// Warp specialisation: warp 4 (the producer) claims items and fills stages
-// with 2-D TMA loads that complete on the stage's `full` mbarrier; warps 0-3
-// wait on `full`, multiply, and arrive on the stage's `empty` mbarrier, which
-// the producer waits on before refilling.  Item epilogues run on the
-// consumers only, so the weight stream never pauses for them.
-//
-// Launched with programmatic stream serialisation: the barrier set-up and
-// the weight boxes of the first item (its index is the CTA index) are issued
-// before griddepcontrol.wait; everything that reads or writes data another
-// kernel touches comes after it.
-template <int NT, bool PAIR>
-struct StreamCfg {
-    static constexpr int kNB = PAIR ? 2 : 4;              // 256-column boxes per stage
-    static constexpr int kCols = 256 * kNB;               // k columns per stage
-    static constexpr int kWarpCols = kCols / 4;           // columns per consumer warp
-    static constexpr int kBoxW = 256 * 16;                // elements of a weight box
-    static constexpr int kARows = 8 * NT;
-    static constexpr int kBoxA = 256 * kARows;            // elements of an activation box
-    static constexpr int kWBlocks = PAIR ? 2 : 1;
-    static constexpr int kStage = kWBlocks * kNB * kBoxW + kNB * kBoxA;  // elements per stage
-    static constexpr uint32_t kBytes = 2u * kStage;
-    static constexpr int kStages = (int)((200u * 1024u) / kBytes) > 8 ? 8 : (int)((200u * 1024u) / kBytes);
-};
-
-template <int NT, bool PAIR>
-static size_t stream_smem() {
-    using C = StreamCfg<NT, PAIR>;
-    return sizeof(__nv_bfloat16) * (size_t)C::kStages * C::kStage + 128;  // + alignment slack
-}
-
-KS_DEV uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
-
-KS_DEV void mbar_init(uint64_t* bar, uint32_t count) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
-}
-KS_DEV void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
-                 : "memory");
-}
-KS_DEV void mbar_arrive(uint64_t* bar) {
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
-}
-KS_DEV void tma_2d(void* dst, const CUtensorMap* map, int x, int y, uint64_t* bar) {
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], "
-        "[%4];" ::"r"(smem_u32(dst)),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar))
-        : "memory");
-}
-KS_DEV void grid_dependency_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
-KS_DEV uint64_t global_ns() {
-    uint64_t t;
-    asm volatile("mov.u64 %0, %globaltimer;" : "=l"(t));
-    return t;
-}
-// Wait for the mbarrier phase with the given parity; gives up after limit_ns.
-KS_DEV bool mbar_wait(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
-    const uint32_t b = smem_u32(bar);
-    uint64_t t0 = 0;
-    for (uint32_t i = 0;; ++i) {
-        uint32_t ok;
-        asm volatile(
-            "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
-            : "=r"(ok)
-            : "r"(b), "r"(parity)
-            : "memory");
-        if (ok) return true;
-        if (i == 0) t0 = global_ns();
-        else if ((i & 63) == 0 && global_ns() - t0 > limit_ns) return false;
-    }
-}
-// Barrier of the four consumer warps that also ORs a flag across them.
-KS_DEV bool consumers_or(bool v) {
-    uint32_t r;
-    asm volatile(
-        "{ .reg .pred p, q; setp.ne.u32 p, %1, 0; bar.red.or.pred q, 1, 128, p; selp.u32 %0, 1, 0, q; }"
-        : "=r"(r)
-        : "r"((uint32_t)v)
-        : "memory");
-    return r != 0;
-}
-
-constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s: only a broken copy waits this long
-
-// Persistent: grid = SM count, one CTA (5 warps) per SM.  CTA b starts with
-// item b, then takes gridDim.x + (ticket from counters[0]); its tiles go
-// through ring slot t % S in order.
-template <int NT, int EPI>
-__global__ void __launch_bounds__(160, 1) gemv_stream_kernel(const __grid_constant__ GemvArgs a) {
-    constexpr bool PAIR = (EPI == EPI_SWIGLU);
-    using Cfg = StreamCfg<NT, PAIR>;
-    constexpr int S = Cfg::kStages;
-    extern __shared__ unsigned char smem_raw[];
-    __nv_bfloat16* stages = reinterpret_cast<__nv_bfloat16*>(
-        (reinterpret_cast<uintptr_t>(smem_raw) + 127) & ~static_cast<uintptr_t>(127));
-    __shared__ __align__(8) uint64_t full[S];
-    __shared__ __align__(8) uint64_t empty[S];
-    __shared__ int slot_item[S];
-    __shared__ int slot_kt[S];
-    __shared__ float scale[kMaxRows];
-    __shared__ float red[3][2][NT * 4][32];   // partial fragments of warps 1-3
-    __shared__ int is_last;
-
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int g = lane >> 2, t4 = lane & 3;
-    const int n_items = div_up(a.N, 16);
-    const int TPI = div_up(a.K, Cfg::kCols);
-
-    if (tid == 0) {
-        for (int i = 0; i < S; ++i) {
-            mbar_init(&full[i], 1);
-            mbar_init(&empty[i], kGemvWarps);
-        }
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    }
-    __syncthreads();
-
-    if (warp == kGemvWarps) {
-        // ------------------------------------------------------ producer
-        if (lane != 0) return;
-        auto load_w = [&](int slot, int it, int kt) {
-            __nv_bfloat16* st = stages + (size_t)slot * Cfg::kStage;
-            const int k0 = kt * Cfg::kCols;
-#pragma unroll
-            for (int b = 0; b < Cfg::kNB; ++b) {
-                tma_2d(st + b * Cfg::kBoxW, &a.wmap, k0 + 256 * b, it * 16, &full[slot]);
-                if (PAIR) tma_2d(st + (Cfg::kNB + b) * Cfg::kBoxW, &a.wmap, k0 + 256 * b, a.N + it * 16, &full[slot]);
-            }
-        };
-        auto load_x = [&](int slot, int kt) {
-            __nv_bfloat16* st = stages + (size_t)slot * Cfg::kStage + Cfg::kWBlocks * Cfg::kNB * Cfg::kBoxW;
-            const int k0 = kt * Cfg::kCols;
-#pragma unroll
-            for (int b = 0; b < Cfg::kNB; ++b) tma_2d(st + b * Cfg::kBoxA, &a.xmap, k0 + 256 * b, 0, &full[slot]);
-        };
-        // bytes landing per stage: the weight boxes plus activation boxes of R rows
-        const uint32_t bytes = 2u * (Cfg::kWBlocks * Cfg::kNB * Cfg::kBoxW + Cfg::kNB * 256 * a.R);
-        // first item (static): weights before the grid dependency resolves
-        int it = blockIdx.x;
-        int t = 0;
-        const int pre = (it < n_items) ? min(S, TPI) : 0;
-        for (int kt = 0; kt < pre; ++kt) {
-            slot_item[kt] = it;
-            slot_kt[kt] = kt;
-            mbar_expect_tx(&full[kt], bytes);
-            load_w(kt, it, kt);
-        }
-        grid_dependency_wait();
-        for (int kt = 0; kt < pre; ++kt) load_x(kt, kt);
-        bool ok = true;
-        int kt0 = pre;
-        t = pre;
-        for (;;) {
-            if (it < n_items) {
-                for (int kt = kt0; kt < TPI; ++kt, ++t) {
-                    const int slot = t % S;
-                    if (t >= S && !mbar_wait(&empty[slot], (uint32_t)(((t / S) - 1) & 1), kWaitLimitNs)) {
-                        ok = false;
-                        break;
-                    }
-                    slot_item[slot] = it;
-                    slot_kt[slot] = kt;
-                    mbar_expect_tx(&full[slot], bytes);
-                    load_w(slot, it, kt);
-                    load_x(slot, kt);
-                }
-                if (!ok) break;
-                it = gridDim.x + atomicAdd(&a.counters[0], 1);
-                kt0 = 0;
-                continue;
-            }
-            // no more work: a sentinel stage tells the consumers
-            const int slot = t % S;
-            if (t >= S && !mbar_wait(&empty[slot], (uint32_t)(((t / S) - 1) & 1), kWaitLimitNs)) {
-                ok = false;
-                break;
-            }
-            slot_item[slot] = -1;
-            mbar_arrive(&full[slot]);
-            break;
-        }
-        if (!ok) atomicExch(a.err, 1);
-        // nothing more to stream: the next kernel may start on SMs as they free up
-        asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-        return;
-    }
-
-    // ---------------------------------------------------------- consumers
-    grid_dependency_wait();
-    if (tid < kMaxRows) {
-        // per-row output scale: 1 / rms(x) from the producer's sums of squares
-        float sc = 1.f;
-        if (a.ss_in != nullptr && tid < a.R) {
-            float ssum = 0.f;
-            for (int q = 0; q < a.ss_groups; ++q) ssum += a.ss_in[q * kMaxRows + tid];
-            sc = rsqrtf(ssum / (float)a.K + a.eps);
-        }
-        scale[tid] = sc;
-    }
-    out_sync<true>();
-
-    const uint4 z = make_uint4(0, 0, 0, 0);
-    // this warp's columns inside a stage: box wb, columns [wc, wc + kWarpCols)
-    const int wb = (warp * Cfg::kWarpCols) / 256, wc = (warp * Cfg::kWarpCols) % 256;
-    float acc[NT][4], accu[NT][4];
-    bool failed = false;
-    for (int t = 0;; ++t) {
-        const int slot = t % S;
-        const bool ok = mbar_wait(&full[slot], (uint32_t)((t / S) & 1), kWaitLimitNs);
-        if (consumers_or(!ok)) {
-            failed = true;
-            break;
-        }
-        const int it = slot_item[slot];
-        if (it < 0) break;
-        const int kt = slot_kt[slot];
-        if (kt == 0) {
-#pragma unroll
-            for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-                for (int i = 0; i < 4; ++i) acc[nt][i] = accu[nt][i] = 0.f;
-        }
-        const __nv_bfloat16* st = stages + (size_t)slot * Cfg::kStage;
-        const __nv_bfloat16* w0p = st + wb * Cfg::kBoxW + g * 256 + wc + 8 * t4;
-        const __nv_bfloat16* ap = st + Cfg::kWBlocks * Cfg::kNB * Cfg::kBoxW + wb * Cfg::kBoxA + g * 256 + wc + 8 * t4;
-#pragma unroll
-        for (int ks = 0; ks < Cfg::kWarpCols / 32; ++ks) {
-            const uint4 w0 = lds128(w0p + 32 * ks);
-            const uint4 w1 = lds128(w0p + 8 * 256 + 32 * ks);
-            uint4 u0 = z, u1 = z;
-            if (PAIR) {
-                u0 = lds128(w0p + Cfg::kNB * Cfg::kBoxW + 32 * ks);
-                u1 = lds128(w0p + Cfg::kNB * Cfg::kBoxW + 8 * 256 + 32 * ks);
-            }
-#pragma unroll
-            for (int nt = 0; nt < NT; ++nt) {
-                const uint4 bv = (nt * 8 + g < a.R) ? lds128(ap + nt * 8 * 256 + 32 * ks) : z;
-                mma_bf16(acc[nt], w0.x, w1.x, w0.y, w1.y, bv.x, bv.y);
-                mma_bf16(acc[nt], w0.z, w1.z, w0.w, w1.w, bv.z, bv.w);
-                if (PAIR) {
-                    mma_bf16(accu[nt], u0.x, u1.x, u0.y, u1.y, bv.x, bv.y);
-                    mma_bf16(accu[nt], u0.z, u1.z, u0.w, u1.w, bv.z, bv.w);
-                }
-            }
-        }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&empty[slot]);  // this warp is done with the stage
-        if (kt != TPI - 1) continue;
-
-        // ------------------------------------------------ item epilogue
-        // warps 1-3 hand their K-quarter partials to warp 0, which adds them
-        // in warp order; the fragment of lane (g, t) covers features
-        // 16 it + g (+ 8) and rows nt * 8 + 2 t (+ 1).
-        if (warp > 0) {
-#pragma unroll
-            for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    red[warp - 1][0][nt * 4 + i][lane] = acc[nt][i];
-                    if (PAIR) red[warp - 1][1][nt * 4 + i][lane] = accu[nt][i];
-                }
-        }
-        out_sync<true>();
-        if (warp == 0) {
-#pragma unroll
-            for (int w = 0; w < 3; ++w)
-#pragma unroll
-                for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-                    for (int i = 0; i < 4; ++i) {
-                        acc[nt][i] += red[w][0][nt * 4 + i][lane];
-                        if (PAIR) accu[nt][i] += red[w][1][nt * 4 + i][lane];
-                    }
-            float ssq[NT][2], bv[NT][2];
-            int bi[NT][2];
-#pragma unroll
-            for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-                for (int c = 0; c < 2; ++c) {
-                    ssq[nt][c] = 0.f;
-                    bv[nt][c] = -INFINITY;
-                    bi[nt][c] = INT_MAX;
-                }
-#pragma unroll
-            for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    const int n = it * 16 + g + 8 * (i >> 1);
-                    const int r = nt * 8 + 2 * t4 + (i & 1);
-                    if (n < a.N && r < a.R) {
-                        const float sc = scale[r];
-                        const float v = acc[nt][i] * sc;
-                        if (EPI == EPI_LMHEAD) {
-                            a.logits[(size_t)r * a.logits_ld + n] = v;
-                            if (better(v, n, bv[nt][i & 1], bi[nt][i & 1])) {
-                                bv[nt][i & 1] = v;
-                                bi[nt][i & 1] = n;
-                            }
-                        } else if (EPI == EPI_RESID) {
-                            float* x = a.resid + (size_t)r * a.resid_ld + n;
-                            const float nx = *x + v;
-                            *x = nx;
-                            if (a.capture) a.capture[(size_t)r * a.capture_ld + n] = nx;
-                            a.xg_out[(size_t)r * a.resid_ld + n] = __float2bfloat16_rn(
-                                nx * to_float(reinterpret_cast<const __nv_bfloat16*>(a.next_gain)[n]));
-                            ssq[nt][i & 1] = fmaf(nx, nx, ssq[nt][i & 1]);
-                        } else {
-                            apply_epilogue<__nv_bfloat16, EPI>(a, n, r, v, accu[nt][i] * sc);
-                        }
-                    }
-                }
-            if (EPI == EPI_RESID || EPI == EPI_LMHEAD) {
-                // reduce over the 8 lanes with the same t (features g, g + 8)
-#pragma unroll
-                for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-                    for (int c = 0; c < 2; ++c) {
-                        const int r = nt * 8 + 2 * t4 + c;
-#pragma unroll
-                        for (int o = 4; o < 32; o <<= 1) {
-                            if (EPI == EPI_RESID) {
-                                ssq[nt][c] += __shfl_xor_sync(0xffffffffu, ssq[nt][c], o);
-                            } else {
-                                const float ov = __shfl_xor_sync(0xffffffffu, bv[nt][c], o);
-                                const int oi = __shfl_xor_sync(0xffffffffu, bi[nt][c], o);
-                                if (better(ov, oi, bv[nt][c], bi[nt][c])) {
-                                    bv[nt][c] = ov;
-                                    bi[nt][c] = oi;
-                                }
-                            }
-                        }
-                        if (g == 0 && r < a.R) {
-                            if (EPI == EPI_RESID) {
-                                a.ss_out[it * kMaxRows + r] = ssq[nt][c];
-                            } else {
-                                a.amax_val[it * kMaxRows + r] = bv[nt][c];
-                                a.amax_idx[it * kMaxRows + r] = bi[nt][c];
-                            }
-                        }
-                    }
-            }
-        }
-        out_sync<true>();  // red[] may be reused
-    }
-    if (failed) {
-        if (tid == 0) atomicExch(a.err, 1);
-        return;  // leave the queue alone; the host sees the status word
-    }
-    // the last CTA to finish resets the queue (every producer has stopped claiming)
-    out_sync<true>();
-    if (tid == 0) {
-        __threadfence();
-        is_last = (atomicAdd(&a.counters[1], 1) == (int)gridDim.x - 1);
-    }
-    out_sync<true>();
-    if (!is_last) return;
-    __threadfence();
-    if (EPI == EPI_LMHEAD) final_argmax(a, n_items);
-    if (tid == 0) {
-        a.counters[0] = 0;
-        a.counters[1] = 0;
-    }
-}
-
 // ---------------------------------------------------------------- launcher
-bool make_tma_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t K, uint32_t box_rows) {
+static PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
     static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
     if (encode == nullptr) {
         void* fn = nullptr;
@@ -764,10 +374,15 @@ bool make_tma_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t K,
         if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) !=
                 cudaSuccess ||
             q != cudaDriverEntryPointSuccess || fn == nullptr)
-            return false;
+            return nullptr;
         encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
     }
-    if (K % 8 != 0 || (reinterpret_cast<uintptr_t>(base) & 15) != 0) return false;
+    return encode;
+}
+
+bool make_tma_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t K, uint32_t box_rows) {
+    auto encode = tensor_map_encoder();
+    if (!encode || K % 8 != 0 || (reinterpret_cast<uintptr_t>(base) & 15) != 0) return false;
     const cuuint64_t dims[2] = {K, rows};
     const cuuint64_t strides[1] = {K * 2};
     const cuuint32_t box[2] = {256, box_rows};
@@ -777,28 +392,41 @@ bool make_tma_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t K,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+bool make_weight_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t K, uint32_t chunks) {
+    auto encode = tensor_map_encoder();
+    if (!encode || K % 8 != 0 || (reinterpret_cast<uintptr_t>(base) & 15) != 0) return false;
+    const cuuint32_t estr[3] = {1, 1, 1};
+    if (K % 64 == 0) {
+        // {64 columns, rows, K / 64 chunks}: a box is `chunks` chunks of 16 rows
+        const cuuint64_t dims[3] = {64, rows, K / 64};
+        const cuuint64_t strides[2] = {K * 2, 128};
+        const cuuint32_t box[3] = {64, 16, chunks};
+        return encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+                      CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                      CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+    }
+    const cuuint64_t dims[2] = {K, rows};
+    const cuuint64_t strides[1] = {K * 2};
+    const cuuint32_t box[2] = {64, 16};
+    return encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
 
-template <int EPI>
-static cudaError_t launch_stream(const GemvArgs& a, cudaStream_t s) {
-    if (a.err == nullptr || a.R > kMaxRows || a.K % 8 != 0) return cudaErrorInvalidValue;
-    auto run = [&](auto kern, size_t smem) -> cudaError_t {
-        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        cudaLaunchConfig_t cfg = {};
-        cfg.gridDim = dim3(sm_count());
-        cfg.blockDim = dim3(160);
-        cfg.dynamicSmemBytes = smem;
-        cfg.stream = s;
-        cudaLaunchAttribute attr[1];
-        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-        attr[0].val.programmaticStreamSerializationAllowed = 1;
-        cfg.attrs = attr;
-        cfg.numAttrs = 1;
-        return cudaLaunchKernelEx(&cfg, kern, a);
-    };
-    constexpr bool PAIR = EPI == EPI_SWIGLU;
-    if (a.R <= 8) return run(gemv_stream_kernel<1, EPI>, stream_smem<1, PAIR>());
-    return run(gemv_stream_kernel<2, EPI>, stream_smem<2, PAIR>());
+bool make_stage_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t K, uint32_t box_rows,
+                    uint32_t chunks) {
+    if (K % 256 != 0) return make_tma_map(map, base, rows, K, box_rows);
+    auto encode = tensor_map_encoder();
+    if (!encode || (reinterpret_cast<uintptr_t>(base) & 15) != 0) return false;
+    // [rows][K] viewed as {256 columns, rows, K / 256 chunks}: one box holds
+    // `chunks` consecutive 256-column chunks of box_rows rows, chunk-major
+    const cuuint64_t dims[3] = {256, rows, K / 256};
+    const cuuint64_t strides[2] = {K * 2, 512};
+    const cuuint32_t box[3] = {256, box_rows, chunks};
+    const cuuint32_t estr[3] = {1, 1, 1};
+    return encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 template <int EPI>
@@ -819,15 +447,8 @@ static cudaError_t launch_f32(const GemvArgs& a, cudaStream_t s) {
 }
 
 cudaError_t launch_gemv(int dtype, int epi, const GemvArgs& a, cudaStream_t s) {
-    if (a.R < 1 || a.R > kMaxRows || a.dtype != dtype) return cudaErrorInvalidValue;
-    if (dtype == 1) {
-        switch (epi) {
-            case EPI_STORE: return launch_stream<EPI_STORE>(a, s);
-            case EPI_RESID: return launch_stream<EPI_RESID>(a, s);
-            case EPI_SWIGLU: return launch_stream<EPI_SWIGLU>(a, s);
-            default: return launch_stream<EPI_LMHEAD>(a, s);
-        }
-    }
+    // fp32 models only; bf16 projections run in the chain kernel
+    if (a.R < 1 || a.R > kMaxRows || a.dtype != dtype || dtype != 0) return cudaErrorInvalidValue;
     switch (epi) {
         case EPI_STORE: return launch_f32<EPI_STORE>(a, s);
         case EPI_RESID: return launch_f32<EPI_RESID>(a, s);

@@ -14,8 +14,6 @@ namespace ks {
 enum GemvEpi { EPI_STORE = 0, EPI_RESID = 1, EPI_SWIGLU = 2, EPI_LMHEAD = 3 };
 
 struct GemvArgs {
-    CUtensorMap wmap;       // bf16: TMA map of W (dims {K, rows}, box 256 x 16)
-    CUtensorMap xmap;       // bf16: TMA map of the input rows (dims {K, max_rows}, box 256 x R)
     int dtype;              // KS_DTYPE_F32 / KS_DTYPE_BF16 (selects kernel and split plan)
     const void* W;          // [N (or 2N for SwiGLU)][K], row stride K, model dtype
     int N;                  // output features (SwiGLU: d_ff; rows n and N + n pair up)
@@ -52,7 +50,54 @@ cudaError_t launch_gemv(int dtype, int epi, const GemvArgs& a, cudaStream_t s);
 // TMA map of a row-major bf16 matrix [rows][K] (K % 8 == 0, 16-byte aligned
 // base), box 256 columns x box_rows rows, no swizzle, zero fill outside.
 bool make_tma_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t K, uint32_t box_rows);
+// Map for the chain kernel's stages: when K % 256 == 0 a 3-D view
+// {256, rows, K / 256} whose box {256, box_rows, chunks} is a whole stage (one
+// copy); otherwise the 2-D map above (one copy per 256-column chunk).
+bool make_stage_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t K, uint32_t box_rows,
+                    uint32_t chunks);
+// Weight map for the chain kernel: 64-column chunks of 16 rows with the
+// 128-byte swizzle (16-byte unit u of row r lands at unit u ^ (r & 7)).
+// K % 64 == 0: 3-D view {64, rows, K / 64}, box of `chunks` chunks (one copy
+// per stage); otherwise 2-D, box {64, 16} (one copy per chunk).
+bool make_weight_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t K, uint32_t chunks);
 int gemv_groups(int N, int dtype);              // output groups (argmax candidates) of a launch
+
+// ----------------------------------------------------------------- chain
+// bf16 models: a run of consecutive projections (phases) in one persistent
+// launch.  Phase codes: 4 l + kind for layer l (kind: ChainKind 0..3), 4 L for
+// the LM head.  Each phase reads the previous phase's complete output.  The
+// tensor maps travel in the kernel parameters (TMA reads them from there
+// without a descriptor fetch from global memory), which bounds a launch to
+// kChainMaxPhases phases (about 24 KB of parameters).
+constexpr int kChainMaxPhases = 160;
+enum ChainKind { CH_QKV = 0, CH_O = 1, CH_GU = 2, CH_DOWN = 3, CH_LM = 4 };
+
+struct ChainArgs {
+    CUtensorMap wmap[kChainMaxPhases];  // weights of each phase (make_weight_map)
+    CUtensorMap amap[4];        // inputs for this R: xg (4-chunk stages), xg (2-chunk), attn_out, act
+    int n_phases;
+    int R;                      // rows, 1..16
+    int stages;                 // ring stages (set by launch_chain)
+    int n_layers, d, F, nqkv, hqd, vocab;
+    float eps;
+    float* x;                   // [R][d] fp32 residual (O / down add into it)
+    float* ss;                  // [d / 16][16] per-16-feature sums of squares of x
+    __nv_bfloat16* xg;          // [R][d] x * gain of the next RMSNorm (input of QKV / gate-up / LM head)
+    float* qkv;                 // [R][nqkv] fp32
+    __nv_bfloat16* act;         // [R][F] silu(gate) * up
+    float* logits;              // [R][vocab]
+    unsigned long long* best;   // [16] LM head argmax keys (zero between launches)
+    int* tokens;                // [R] LM head argmax
+    float* capture;             // history capture or null: sublayer i's rows at capture + i * capture_plane
+    long long capture_plane;
+    int* counters;              // chain_counter_ints() zeros; the launch leaves them zero
+    int* err;                   // device status word
+    uint16_t code[kChainMaxPhases];
+    const __nv_bfloat16* gain[kChainMaxPhases];  // O / down phases: gain of the next RMSNorm
+};
+size_t chain_counter_ints();
+cudaError_t launch_chain(const ChainArgs& a, cudaStream_t s);
+int sm_count();
 
 // ------------------------------------------------------------- attention
 struct AttnArgs {

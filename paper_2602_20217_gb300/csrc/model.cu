@@ -35,8 +35,8 @@ cudaError_t launch_select(const ks_latency* lat, const float* sims, int64_t n, i
                           int32_t* budget_out, void* scratch, int cap, cudaStream_t s);
 
 constexpr int kSelectCap = 65535;
-constexpr int kKlasses = 9;
-enum { K_QKV = 0, K_ATTN, K_MERGE, K_OPROJ, K_GATEUP, K_DOWN, K_LMHEAD, K_EMBED, K_ACCEPT };
+constexpr int kKlasses = 10;
+enum { K_QKV = 0, K_ATTN, K_MERGE, K_OPROJ, K_GATEUP, K_DOWN, K_LMHEAD, K_EMBED, K_ACCEPT, K_CHAIN };
 
 // ------------------------------------------------------------ small kernels
 // x[r] = embed[tok[r]] (fp32); optionally copied to the history plane 0.
@@ -86,7 +86,7 @@ static size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
 struct Layout {
     size_t kv, rope, x, ss, xg, qkv, attn_out, act, attn_part, gemv_part, counters, logits, amax_val,
-        amax_idx, tok, hist, hist_snap, hist_idx, sims, mask, obj, wts, select, total;
+        amax_idx, tok, hist, hist_snap, hist_idx, sims, mask, obj, wts, select, chain_ctr, best, total;
     int n_chunks_max;
     size_t gemv_part_floats;
     int counters_n;
@@ -161,6 +161,9 @@ static Layout make_layout(const ks_config* c) {
     L.obj = take(sizeof(double) * 2);
     L.wts = take(sizeof(int) * (nsub + 2));
     L.select = take(select_scratch_bytes(nsub, kSelectCap));
+    // bf16: two sets of chain counters
+    L.chain_ctr = take(sizeof(int) * 2 * chain_counter_ints());
+    L.best = take(sizeof(unsigned long long) * 16);
     L.total = off;
     return L;
 }
@@ -173,6 +176,7 @@ struct KlassTiming {
     bool on = false;
     std::vector<cudaEvent_t> ev;  // pairs
     size_t used = 0;
+    double bytes = 0.0;           // weight bytes the timed launches had to stream
 };
 
 struct ks_model {
@@ -195,6 +199,10 @@ struct ks_model {
     void *attn_out, *act, *select;
     int *counters, *amax_idx, *rows, *target, *result, *err, *seq, *hist_idx;
     uint8_t* mask_dev;
+    ChainArgs* chain = nullptr;  // bf16: parameter block of the chain launches (host)
+    int* chain_ctr;           // two counter sets, alternating between chain launches
+    unsigned long long* best; // LM head argmax keys of the chain kernel
+    int chain_parity = 0;
     double* obj_dev;
     int* wts_dev;
     // pinned host staging
@@ -215,7 +223,7 @@ struct ks_model {
     int64_t h2d = 0, d2h = 0;
     // bf16: TMA maps of every weight matrix and of the three projection inputs
     std::vector<CUtensorMap> map_qkv, map_o, map_gu, map_down;
-    CUtensorMap map_lm, map_xg[16], map_attn_out[16], map_act[16];  // [R - 1]: boxes of exactly R rows
+    CUtensorMap map_lm, map_xg[16], map_xg2[16], map_attn_out[16], map_act[16];  // [R - 1]: boxes of R rows
     KlassTiming timing[kKlasses];
 };
 
@@ -232,8 +240,9 @@ static ks_status cuda_fail(cudaError_t e, const char* what) {
     } while (0)
 
 template <class F>
-static ks_status launch(ks_model* m, int klass, F&& f, const char* what) {
+static ks_status launch(ks_model* m, int klass, F&& f, const char* what, double bytes = 0.0) {
     KlassTiming& T = m->timing[klass];
+    if (T.on) T.bytes += bytes;
     cudaEvent_t e0 = nullptr, e1 = nullptr;
     if (T.on) {
         if (T.used + 2 > T.ev.size()) {
@@ -347,39 +356,113 @@ static ks_status forward(ks_model* m, const int32_t* tok, int R, int p0, const u
         return cudaGetLastError();
     }, "embed"));
 
+    // attention core of layer l: RoPE / QK-norm, cache write, split-KV, merge
+    auto attention = [&](int l) -> ks_status {
+        AttnArgs at{};
+        at.qkv = m->qkv; at.qkv_ld = nqkv; at.R = R; at.p0 = p0;
+        at.hq = c.n_q_heads; at.hk = c.n_kv_heads; at.hd = hd;
+        at.kcache = kcache(m, l); at.vcache = vcache(m, l); at.max_seq = c.max_seq;
+        at.rope = m->rope;
+        at.q_norm = c.qk_norm ? m->q_norm[l] : nullptr;
+        at.k_norm = c.qk_norm ? m->k_norm[l] : nullptr;
+        at.eps = c.rms_eps;
+        at.part = m->attn_part; at.n_chunks_max = m->lay.n_chunks_max;
+        at.out = m->attn_out; at.out_ld = c.n_q_heads * hd;
+        KS_TRY(launch(m, K_ATTN, [&] { return launch_attention(dt, at, s); }, "attention"));
+        KS_TRY(launch(m, K_MERGE, [&] { return launch_attn_merge(dt, at, s); }, "attention merge"));
+        return KS_OK;
+    };
     for (int l = 0; l < c.n_layers; ++l) {
-        const bool run_attn = runs(2 * l + 1);
-        const bool run_mlp = runs(2 * l + 2);
-        if ((!run_attn || !run_mlp) && capture_slot >= 0) {
+        if ((!runs(2 * l + 1) || !runs(2 * l + 2)) && capture_slot >= 0) {
             set_error("forward: capture needs every sublayer");
             return KS_ERR_STATE;
         }
+    }
+
+    if (bf) {
+        // bf16: consecutive projections run as one chain launch; a chain ends
+        // at each attention core.  While a projection class is being timed,
+        // every projection is its own launch so that it can be timed alone.
+        const bool split = m->timing[K_QKV].on || m->timing[K_OPROJ].on || m->timing[K_GATEUP].on ||
+                           m->timing[K_DOWN].on || m->timing[K_LMHEAD].on;
+        const int L = c.n_layers, F = c.d_ff, hqd = c.n_q_heads * hd;
+        if (!m->chain) m->chain = new ChainArgs();
+        ChainArgs& ca = *m->chain;
+        ca.amap[0] = m->map_xg[R - 1];
+        ca.amap[1] = m->map_xg2[R - 1];
+        ca.amap[2] = m->map_attn_out[R - 1];
+        ca.amap[3] = m->map_act[R - 1];
+        ca.R = R;
+        ca.n_layers = L; ca.d = d; ca.F = F; ca.nqkv = nqkv; ca.hqd = hqd; ca.vocab = c.vocab;
+        ca.eps = c.rms_eps;
+        ca.x = m->x; ca.ss = m->ss; ca.xg = m->xg; ca.qkv = m->qkv;
+        ca.act = reinterpret_cast<__nv_bfloat16*>(m->act);
+        ca.logits = m->logits; ca.best = m->best; ca.tokens = argmax;
+        ca.capture = capture_slot >= 0 ? hist_plane(m, 0) + (size_t)capture_slot * c.max_rows * d : nullptr;
+        ca.capture_plane = (long long)m->lay.hist_slots * c.max_rows * d;
+        ca.err = m->err;
+        int nph = 0, klass = K_CHAIN;
+        double bytes = 0.0;
+        auto flush = [&]() -> ks_status {
+            if (nph == 0) return KS_OK;
+            ca.n_phases = nph;
+            ca.counters = m->chain_ctr + (size_t)m->chain_parity * chain_counter_ints();
+            m->chain_parity ^= 1;
+            KS_TRY(launch(m, split ? klass : K_CHAIN, [&] { return launch_chain(ca, s); }, "projections", bytes));
+            nph = 0;
+            bytes = 0.0;
+            return KS_OK;
+        };
+        auto add = [&](int layer, int kind, const void* gain, int k_class) -> ks_status {
+            const double es2 = 2.0;
+            const double wb = kind == CH_QKV ? es2 * nqkv * d
+                            : kind == CH_O ? es2 * d * hqd
+                            : kind == CH_GU ? es2 * 2.0 * F * d
+                            : kind == CH_DOWN ? es2 * d * F
+                            : es2 * c.vocab * d;
+            ca.code[nph] = (uint16_t)(kind == CH_LM ? 4 * L : 4 * layer + kind);
+            ca.gain[nph] = reinterpret_cast<const __nv_bfloat16*>(gain);
+            ca.wmap[nph] = kind == CH_QKV ? m->map_qkv[layer]
+                         : kind == CH_O ? m->map_o[layer]
+                         : kind == CH_GU ? m->map_gu[layer]
+                         : kind == CH_DOWN ? m->map_down[layer] : m->map_lm;
+            ++nph;
+            bytes += wb;
+            klass = k_class;
+            return (split || nph == kChainMaxPhases) ? flush() : KS_OK;
+        };
+        for (int l = 0; l < L; ++l) {
+            if (runs(2 * l + 1)) {
+                KS_TRY(add(l, CH_QKV, nullptr, K_QKV));
+                KS_TRY(flush());
+                KS_TRY(attention(l));
+                KS_TRY(add(l, CH_O, next_gain(2 * l + 1), K_OPROJ));
+            }
+            if (runs(2 * l + 2)) {
+                KS_TRY(add(l, CH_GU, nullptr, K_GATEUP));
+                KS_TRY(add(l, CH_DOWN, next_gain(2 * l + 2), K_DOWN));
+            }
+        }
+        if (argmax) KS_TRY(add(0, CH_LM, nullptr, K_LMHEAD));
+        KS_TRY(flush());
+        m->last_pass_rows = R;
+        return KS_OK;
+    }
+
+    for (int l = 0; l < c.n_layers; ++l) {
+        const bool run_attn = runs(2 * l + 1);
+        const bool run_mlp = runs(2 * l + 2);
         if (run_attn) {
             GemvArgs g{};
             common(g, m->w_qkv[l], nqkv, d);
             norm_input(g, m->attn_norm[l]);
-            if (bf) { g.wmap = m->map_qkv[l]; g.xmap = m->map_xg[R - 1]; }
             g.out = m->qkv;
             g.out_ld = nqkv;
             gemv_plan(g, EPI_STORE);
             KS_TRY(launch(m, K_QKV, [&] { return launch_gemv(dt, EPI_STORE, g, s); }, "qkv"));
-
-            AttnArgs at{};
-            at.qkv = m->qkv; at.qkv_ld = nqkv; at.R = R; at.p0 = p0;
-            at.hq = c.n_q_heads; at.hk = c.n_kv_heads; at.hd = hd;
-            at.kcache = kcache(m, l); at.vcache = vcache(m, l); at.max_seq = c.max_seq;
-            at.rope = m->rope;
-            at.q_norm = c.qk_norm ? m->q_norm[l] : nullptr;
-            at.k_norm = c.qk_norm ? m->k_norm[l] : nullptr;
-            at.eps = c.rms_eps;
-            at.part = m->attn_part; at.n_chunks_max = m->lay.n_chunks_max;
-            at.out = m->attn_out; at.out_ld = c.n_q_heads * hd;
-            KS_TRY(launch(m, K_ATTN, [&] { return launch_attention(dt, at, s); }, "attention"));
-            KS_TRY(launch(m, K_MERGE, [&] { return launch_attn_merge(dt, at, s); }, "attention merge"));
-
+            KS_TRY(attention(l));
             GemvArgs o{};
             common(o, m->w_o[l], d, c.n_q_heads * hd);
-            if (bf) { o.wmap = m->map_o[l]; o.xmap = m->map_attn_out[R - 1]; }
             o.in = m->attn_out;
             o.in_ld = c.n_q_heads * hd;
             resid_output(o, 2 * l + 1);
@@ -390,15 +473,12 @@ static ks_status forward(ks_model* m, const int32_t* tok, int R, int p0, const u
             GemvArgs gu{};
             common(gu, m->w_gate_up[l], c.d_ff, d);
             norm_input(gu, m->mlp_norm[l]);
-            if (bf) { gu.wmap = m->map_gu[l]; gu.xmap = m->map_xg[R - 1]; }
             gu.act = m->act;
             gu.act_ld = c.d_ff;
             gemv_plan(gu, EPI_SWIGLU);
             KS_TRY(launch(m, K_GATEUP, [&] { return launch_gemv(dt, EPI_SWIGLU, gu, s); }, "gate-up"));
-
             GemvArgs dn{};
             common(dn, m->w_down[l], d, c.d_ff);
-            if (bf) { dn.wmap = m->map_down[l]; dn.xmap = m->map_act[R - 1]; }
             dn.in = m->act;
             dn.in_ld = c.d_ff;
             resid_output(dn, 2 * l + 2);
@@ -410,7 +490,6 @@ static ks_status forward(ks_model* m, const int32_t* tok, int R, int p0, const u
         GemvArgs lm{};
         common(lm, m->lm_head, c.vocab, d);
         norm_input(lm, m->final_norm);
-        if (bf) { lm.wmap = m->map_lm; lm.xmap = m->map_xg[R - 1]; }
         lm.logits = m->logits;
         lm.logits_ld = c.vocab;
         lm.amax_val = m->amax_val;
@@ -550,6 +629,8 @@ ks_status ks_model_create(const ks_config* cfg, const ks_weights* w, void* works
     m->hist_idx = reinterpret_cast<int*>(b + lay.hist_idx);
     m->sims = reinterpret_cast<float*>(b + lay.sims);
     m->mask_dev = reinterpret_cast<uint8_t*>(b + lay.mask);
+    m->chain_ctr = reinterpret_cast<int*>(b + lay.chain_ctr);
+    m->best = reinterpret_cast<unsigned long long*>(b + lay.best);
     m->obj_dev = reinterpret_cast<double*>(b + lay.obj);
     m->wts_dev = reinterpret_cast<int*>(b + lay.wts);
     m->select = b + lay.select;
@@ -564,16 +645,17 @@ ks_status ks_model_create(const ks_config* cfg, const ks_weights* w, void* works
         m->map_gu.resize(L);
         m->map_down.resize(L);
         for (int l = 0; l < L && ok; ++l) {
-            ok = ok && make_tma_map(&m->map_qkv[l], m->w_qkv[l], nqkv, d, 16);
-            ok = ok && make_tma_map(&m->map_o[l], m->w_o[l], d, hqd, 16);
-            ok = ok && make_tma_map(&m->map_gu[l], m->w_gate_up[l], 2 * (uint64_t)F, d, 16);
-            ok = ok && make_tma_map(&m->map_down[l], m->w_down[l], d, F, 16);
+            ok = ok && make_weight_map(&m->map_qkv[l], m->w_qkv[l], nqkv, d, 16);
+            ok = ok && make_weight_map(&m->map_o[l], m->w_o[l], d, hqd, 16);
+            ok = ok && make_weight_map(&m->map_gu[l], m->w_gate_up[l], 2 * (uint64_t)F, d, 8);
+            ok = ok && make_weight_map(&m->map_down[l], m->w_down[l], d, F, 16);
         }
-        ok = ok && make_tma_map(&m->map_lm, m->lm_head, cfg->vocab, d, 16);
+        ok = ok && make_weight_map(&m->map_lm, m->lm_head, cfg->vocab, d, 16);
         for (int b = 0; b < R; ++b) {
-            ok = ok && make_tma_map(&m->map_xg[b], m->xg, R, d, b + 1);
-            ok = ok && make_tma_map(&m->map_attn_out[b], m->attn_out, R, hqd, b + 1);
-            ok = ok && make_tma_map(&m->map_act[b], m->act, R, F, b + 1);
+            ok = ok && make_stage_map(&m->map_xg[b], m->xg, R, d, b + 1, 4);
+            ok = ok && make_stage_map(&m->map_xg2[b], m->xg, R, d, b + 1, 2);
+            ok = ok && make_stage_map(&m->map_attn_out[b], m->attn_out, R, hqd, b + 1, 4);
+            ok = ok && make_stage_map(&m->map_act[b], m->act, R, F, b + 1, 4);
         }
         if (!ok) {
             set_error("ks_model_create: TMA descriptor encoding failed");
@@ -614,6 +696,10 @@ ks_status ks_model_create(const ks_config* cfg, const ks_weights* w, void* works
     }
     e = cudaMemsetAsync(m->counters, 0, sizeof(int) * lay.counters_n, m->stream);
     if (e != cudaSuccess) return fail(e, "counter reset");
+    e = cudaMemsetAsync(m->chain_ctr, 0, sizeof(int) * 2 * chain_counter_ints(), m->stream);
+    if (e != cudaSuccess) return fail(e, "counter reset");
+    e = cudaMemsetAsync(m->best, 0, sizeof(unsigned long long) * 16, m->stream);
+    if (e != cudaSuccess) return fail(e, "counter reset");
     e = cudaMemsetAsync(b + lay.tok, 0, sizeof(int) * ((size_t)3 * R + 8 + cfg->max_seq), m->stream);  // incl. err
     if (e != cudaSuccess) return fail(e, "token reset");
     e = cudaStreamSynchronize(m->stream);
@@ -628,6 +714,7 @@ ks_status ks_model_destroy(ks_model* m) {
     for (auto& T : m->timing)
         for (auto e : T.ev) cudaEventDestroy(e);
     if (m->h_buf) cudaFreeHost(m->h_buf);
+    delete m->chain;
     delete m;
     return KS_OK;
 }
@@ -1022,6 +1109,13 @@ ks_status ks_kernel_timing(ks_model* m, int32_t klass, int32_t enable) {
     KS_TRY(sync(m, "timing"));
     m->timing[klass].on = enable != 0;
     m->timing[klass].used = 0;
+    m->timing[klass].bytes = 0.0;
+    return KS_OK;
+}
+
+ks_status ks_kernel_bytes(const ks_model* m, int32_t klass, double* bytes) {
+    if (!m || klass < 0 || klass >= kKlasses || !bytes) return KS_ERR_INVALID_ARG;
+    *bytes = m->timing[klass].bytes;
     return KS_OK;
 }
 

@@ -19,7 +19,7 @@ KS_OK, KS_ERR_INVALID_ARG, KS_ERR_CUDA, KS_ERR_WORKSPACE, KS_ERR_CAPACITY, KS_ER
     KS_ERR_UNSUPPORTED, KS_ERR_STATE = range(8)
 KS_DTYPE_F32, KS_DTYPE_BF16 = 0, 1
 KLASS = {"qkv": 0, "attn": 1, "merge": 2, "oproj": 3, "gateup": 4, "down": 5, "lmhead": 6,
-         "embed": 7, "accept": 8}
+         "embed": 7, "accept": 8, "chain": 9}
 
 
 class KsConfig(C.Structure):
@@ -88,6 +88,7 @@ _SIGS = {
     "ks_debug_read": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32, C.c_int32, C.c_int32, C.c_void_p, C.c_size_t]),
     "ks_kernel_timing": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32]),
     "ks_kernel_time": (C.c_int, [C.c_void_p, C.c_int32, C.POINTER(C.c_int64), C.POINTER(C.c_double)]),
+    "ks_kernel_bytes": (C.c_int, [C.c_void_p, C.c_int32, C.POINTER(C.c_double)]),
     "ks_launch_count": (C.c_int64, [C.c_void_p]),
     "ks_transfer_bytes": (C.c_int, [C.c_void_p, C.POINTER(C.c_int64), C.POINTER(C.c_int64)]),
     "ks_status_str": (C.c_char_p, [C.c_int]),
@@ -292,6 +293,12 @@ def ks_kernel_time(h: int, klass: int):
     n, ms = C.c_int64(), C.c_double()
     check(load().ks_kernel_time(h, klass, C.byref(n), C.byref(ms)), "ks_kernel_time")
     return n.value, ms.value
+
+
+def ks_kernel_bytes(h: int, klass: int) -> float:
+    b = C.c_double()
+    check(load().ks_kernel_bytes(h, klass, C.byref(b)), "ks_kernel_bytes")
+    return b.value
 
 
 def ks_launch_count(h: int) -> int:

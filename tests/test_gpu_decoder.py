@@ -271,3 +271,44 @@ def test_rewind_reuses_the_prompt():
         out, st, acc = m.generate(40, 4, latency=lat, budget_frac=0.6, resolve_every=1)
         assert list(out) == list(spec[0]) and np.array_equal(acc, spec[2])
     m.close()
+
+
+@pytest.mark.parametrize("hd,qk_norm,L", [(128, True, 3), (64, False, 2)])
+def test_chained_projections_equal_one_launch_per_projection(hd, qk_norm, L):
+    """bf16 projections run chained (one persistent launch between attention
+    cores, phases synchronised on device counters) or one per launch (while a
+    projection class is timed).  Both must give bit-identical results: drafts
+    with skipped sublayers (chains across layers), verify with history
+    capture, logits, KV cache and history."""
+    from paper_2602_20217_gb300 import knapspec as ks
+    from paper_2602_20217_gb300 import synth
+    shape = small_bf16(hd, qk_norm, L)
+    prompt = synth.prompt_tokens(shape, 290, seed=5)
+    n = shape.n_sublayers
+    masks = [np.ones(n, np.uint8), np.array([0, 1] * L, np.uint8),
+             np.array(([1, 1, 0, 0] * L)[:n], np.uint8)]
+    runs = []
+    for split in (False, True):
+        m = make(shape, 512)
+        if split:
+            ks.ks_kernel_timing(m.h, ks.KLASS["gateup"], True)
+        m.prefill(prompt)
+        rec = []
+        for mask in masks:
+            d = m.draft(mask, 4)
+            rec.append(("draft", d.copy(), m.logits(1).copy()))
+            a, new = m.verify(None, 4)
+            rec.append(("verify", a, np.array(new), m.logits(5).copy()))
+        rec.append(("hist", m.history().copy()))
+        rec.append(("k", m.kv(L - 1, 0, 300, "k").copy()))
+        rec.append(("greedy", m.decode_greedy(6)))
+        runs.append(rec)
+        if split:
+            nl, ms = ks.ks_kernel_time(m.h, ks.KLASS["gateup"])
+            assert nl > 0 and ms > 0
+            assert ks.ks_kernel_bytes(m.h, ks.KLASS["gateup"]) == nl * 2 * shape.d_ff * shape.d_model * 2
+        m.close()
+    for x, y in zip(*runs):
+        assert x[0] == y[0]
+        for u, v in zip(x[1:], y[1:]):
+            assert np.array_equal(np.asarray(u), np.asarray(v)), x[0]
