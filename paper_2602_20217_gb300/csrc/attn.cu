@@ -18,6 +18,9 @@
 // mma.sync.m16n8k16 with an fp32 online softmax in the log2 domain over the
 // whole chunk.  fp32 models: CUDA-core dot products.  Partials (m, l, o) per
 // (row, query head, chunk) are merged by attn_merge_kernel in a fixed order.
+// bf16 launches use programmatic dependent launch: the attention kernel loads
+// its first tile of old keys before waiting for the projections that produce
+// its queries, and both kernels let their successor launch early.
 #include "common.cuh"
 #include "internal.h"
 
@@ -205,9 +208,9 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const AttnArgs a) {
     __nv_bfloat16* Qs = reinterpret_cast<__nv_bfloat16*>(smem);
     __nv_bfloat16* KV = Qs + (size_t)mpad * P;  // stage s: K at KV + s*2*KT*P, V after it
 
-    // 1. new K/V rows of this chunk -> cache (generic stores, then barrier)
-    write_new_kv<__nv_bfloat16, NPL>(a, h, cs, ce);
-    __syncthreads();
+    // The merge kernel may launch now; it reads the partials only after this
+    // grid completes.
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
     const __nv_bfloat16* kg = reinterpret_cast<const __nv_bfloat16*>(a.kcache) + (size_t)h * a.max_seq * HD;
     const __nv_bfloat16* vg = reinterpret_cast<const __nv_bfloat16*>(a.vcache) + (size_t)h * a.max_seq * HD;
@@ -225,7 +228,17 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const AttnArgs a) {
         }
         cp_async_commit();
     };
-    load_tile(0);
+    // Keys before p0 were written by earlier launches (complete before the
+    // projections that precede this kernel could start), so a first tile of
+    // old keys goes out before waiting for the projections.
+    const bool early = cs + KT <= a.p0;
+    if (early) load_tile(0);
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+
+    // 1. new K/V rows of this chunk -> cache (generic stores, then barrier)
+    write_new_kv<__nv_bfloat16, NPL>(a, h, cs, ce);
+    __syncthreads();
+    if (!early) load_tile(0);
 
     // 2. queries: m = r * G + gq, scaled into the log2 domain, bf16
     const float qscale = kLog2e * rsqrtf((float)HD);
@@ -480,6 +493,8 @@ __global__ void __launch_bounds__(128) attn_merge_kernel(const AttnArgs a) {
     __shared__ float osh[kAttnWarps][HD];
     const int hq_idx = blockIdx.x, r = blockIdx.y;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");   // the next projections may launch
+    asm volatile("griddepcontrol.wait;" ::: "memory");                // the partials are complete
     const int pos = a.p0 + r;
     const int nch = attn_chunk_of(pos) + 1;
     constexpr int S = HD + kPartPad;
@@ -543,8 +558,17 @@ cudaError_t launch_attention(int dtype, const AttnArgs& a, cudaStream_t s) {
         auto run = [&](auto kern) -> cudaError_t {
             cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
             if (e != cudaSuccess) return e;
-            kern<<<grid, 128, smem, s>>>(a);
-            return cudaGetLastError();
+            cudaLaunchConfig_t cfg = {};
+            cfg.gridDim = grid;
+            cfg.blockDim = dim3(128);
+            cfg.dynamicSmemBytes = smem;
+            cfg.stream = s;
+            cudaLaunchAttribute attr[1];
+            attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+            attr[0].val.programmaticStreamSerializationAllowed = 1;
+            cfg.attrs = attr;
+            cfg.numAttrs = 1;
+            return cudaLaunchKernelEx(&cfg, kern, a);
         };
         if (a.hd == 128) return run(attn_bf16_kernel<128>);
         if (a.hd == 64) return run(attn_bf16_kernel<64>);
@@ -568,8 +592,18 @@ cudaError_t launch_attn_merge(int dtype, const AttnArgs& a, cudaStream_t s) {
     const size_t smem = sizeof(float) * (size_t)nch;
     if (smem > 48 * 1024) return cudaErrorInvalidValue;
     if (dtype == 1) {
-        if (a.hd == 128) attn_merge_kernel<__nv_bfloat16, 128><<<grid, 128, smem, s>>>(a);
-        else attn_merge_kernel<__nv_bfloat16, 64><<<grid, 128, smem, s>>>(a);
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = grid;
+        cfg.blockDim = dim3(128);
+        cfg.dynamicSmemBytes = smem;
+        cfg.stream = s;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        if (a.hd == 128) return cudaLaunchKernelEx(&cfg, attn_merge_kernel<__nv_bfloat16, 128>, a);
+        return cudaLaunchKernelEx(&cfg, attn_merge_kernel<__nv_bfloat16, 64>, a);
     } else {
         if (a.hd == 128) attn_merge_kernel<float, 128><<<grid, 128, smem, s>>>(a);
         else attn_merge_kernel<float, 64><<<grid, 128, smem, s>>>(a);
