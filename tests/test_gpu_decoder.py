@@ -32,6 +32,15 @@ def small_bf16(hd=128, qk_norm=False, L=2):
                       dtype="bf16", rope_theta=500000.0)
 
 
+def wide_bf16(L=2):
+    """d 1536 and d_ff 3584: the gate/up (3 stages) and down (4 stages, ragged
+    last stage) projections run as K-sliced items whose partial sums meet in
+    global memory."""
+    from paper_2602_20217_gb300.configs import ModelShape
+    return ModelShape("wide-bf16", L, 1536, 12, 4, 128, 3584, 2000, qk_norm=True, dtype="bf16",
+                      rope_theta=500000.0)
+
+
 def make(shape, max_seq, seed=0):
     from paper_2602_20217_gb300.model import Model
     return Model(shape, max_seq=max_seq, seed=seed)
@@ -175,10 +184,10 @@ def test_tiny_lossless_and_knapsack_policy(tiny):
 
 
 # ------------------------------------------------------------- small bf16
-@pytest.mark.parametrize("hd,qk_norm", [(128, False), (128, True), (64, True)])
+@pytest.mark.parametrize("hd,qk_norm", [(128, False), (128, True), (64, True), ("wide", True)])
 def test_bf16_logits_tokens_and_lossless(hd, qk_norm):
     from paper_2602_20217_gb300 import synth
-    shape = small_bf16(hd, qk_norm)
+    shape = wide_bf16() if hd == "wide" else small_bf16(hd, qk_norm)
     prompt = synth.prompt_tokens(shape, 300, seed=1)
     cfg, w = oracle_model(shape, seed=0)
     m = make(shape, 512)
@@ -273,7 +282,7 @@ def test_rewind_reuses_the_prompt():
     m.close()
 
 
-@pytest.mark.parametrize("hd,qk_norm,L", [(128, True, 3), (64, False, 2)])
+@pytest.mark.parametrize("hd,qk_norm,L", [(128, True, 3), (64, False, 2), ("wide", True, 2)])
 def test_chained_projections_equal_one_launch_per_projection(hd, qk_norm, L):
     """bf16 projections run chained (one persistent launch between attention
     cores, phases synchronised on device counters) or one per launch (while a
@@ -282,7 +291,7 @@ def test_chained_projections_equal_one_launch_per_projection(hd, qk_norm, L):
     capture, logits, KV cache and history."""
     from paper_2602_20217_gb300 import knapspec as ks
     from paper_2602_20217_gb300 import synth
-    shape = small_bf16(hd, qk_norm, L)
+    shape = wide_bf16(L) if hd == "wide" else small_bf16(hd, qk_norm, L)
     prompt = synth.prompt_tokens(shape, 290, seed=5)
     n = shape.n_sublayers
     masks = [np.ones(n, np.uint8), np.array([0, 1] * L, np.uint8),
