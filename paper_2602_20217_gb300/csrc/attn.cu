@@ -13,10 +13,11 @@
 // Per CTA: the new rows' K (QK-RMSNorm, RoPE) and V are written to the cache
 // by the CTA whose chunk holds their position; the G x R query vectors are
 // normalised, rotated and pre-scaled by log2(e)/sqrt(hd).  bf16 models: K/V
-// tiles of 64 keys are double-buffered in shared memory with cp.async; each
-// warp owns a 16-row query tile and runs S = Q K^T and O += P V on
-// mma.sync.m16n8k16 with an fp32 online softmax in the log2 domain over the
-// whole chunk.  fp32 models: CUDA-core dot products.  Partials (m, l, o) per
+// tiles of 64 keys stream through a cp.async ring; for up to two 16-row query
+// tiles at a time the four warps split each tile (warp w: Q K^T for keys
+// 16 w.., P V for head dims w HD/4..) on mma.sync.m16n8k16, with an fp32
+// online softmax in the log2 domain over the whole chunk whose row maxima and
+// sums are combined across warps in warp order.  fp32 models: CUDA-core dot products.  Partials (m, l, o) per
 // (row, query head, chunk) are merged by attn_merge_kernel in a fixed order.
 // bf16 launches use programmatic dependent launch: the attention kernel loads
 // its first tile of old keys before waiting for the projections that produce
@@ -29,6 +30,15 @@ namespace ks {
 constexpr int kAttnWarps = 4;
 constexpr int kPartPad = 4;  // partial row: m, l, 2 pad, o[hd] (16-byte aligned o)
 constexpr int kKeyTile = 64;
+constexpr int kKvStages = 3;   // bf16: K/V tiles in the cp.async ring (two in flight while computing)
+
+// bf16 K/V tiles in shared memory: rows of HD elements, no padding; the
+// 16-byte chunk c of row r is stored at chunk c ^ (r & 7), so the eight rows
+// an ldmatrix reads hit eight different bank groups.
+template <int HD>
+KS_DEV int kv_off(int row, int col) {
+    return row * HD + ((((col >> 3) ^ (row & 7)) << 3) | (col & 7));
+}
 constexpr float kLog2e = 1.4426950408889634f;
 
 // ------------------------------------------------------------ chunk schedule
@@ -185,7 +195,8 @@ KS_DEV int my_chunk(const AttnArgs& a) {
 
 // ----------------------------------------------------------- bf16 kernel
 // Shared layout (bf16, row pitch hd + 8 elements = 16 B padding):
-//   Qs [mpad][P], then 2 stages of { Ks [64][P], Vs [64][P] }.
+//   Qs [mpad][P], then kKvStages stages of { Ks [64][HD], Vs [64][HD] }
+//   (K / V rows unpadded and chunk-swizzled, see kv_off).
 template <int HD>
 __global__ void __launch_bounds__(128) attn_bf16_kernel(const AttnArgs a) {
     constexpr int NPL = HD / 32;
@@ -206,7 +217,7 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const AttnArgs a) {
     const int ntiles = (ce - cs + KT - 1) / KT;
 
     __nv_bfloat16* Qs = reinterpret_cast<__nv_bfloat16*>(smem);
-    __nv_bfloat16* KV = Qs + (size_t)mpad * P;  // stage s: K at KV + s*2*KT*P, V after it
+    __nv_bfloat16* KV = Qs + (size_t)mpad * P;  // stage s: K at KV + s*2*KT*HD, V after it
 
     // The merge kernel may launch now; it reads the partials only after this
     // grid completes.
@@ -216,29 +227,30 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const AttnArgs a) {
     const __nv_bfloat16* vg = reinterpret_cast<const __nv_bfloat16*>(a.vcache) + (size_t)h * a.max_seq * HD;
     constexpr int CPR = HD / 8;  // 16-byte pieces per row
     auto load_tile = [&](int ti) {
-        __nv_bfloat16* Ks = KV + (size_t)(ti & 1) * 2 * KT * P;
-        __nv_bfloat16* Vs = Ks + (size_t)KT * P;
+        __nv_bfloat16* Ks = KV + (size_t)(ti % kKvStages) * 2 * KT * HD;
+        __nv_bfloat16* Vs = Ks + (size_t)KT * HD;
         const int k0 = cs + ti * KT;
         for (int i = tid; i < KT * CPR; i += blockDim.x) {
             const int row = i / CPR, col = (i - row * CPR) * 8;
             const bool ok = k0 + row < ce;
             const size_t off = ok ? (size_t)(k0 + row) * HD + col : 0;
-            cp_async16(Ks + row * P + col, kg + off, ok);
-            cp_async16(Vs + row * P + col, vg + off, ok);
+            cp_async16(Ks + kv_off<HD>(row, col), kg + off, ok);
+            cp_async16(Vs + kv_off<HD>(row, col), vg + off, ok);
         }
         cp_async_commit();
     };
     // Keys before p0 were written by earlier launches (complete before the
-    // projections that precede this kernel could start), so a first tile of
-    // old keys goes out before waiting for the projections.
-    const bool early = cs + KT <= a.p0;
-    if (early) load_tile(0);
+    // projections that precede this kernel could start), so the first tiles
+    // of old keys go out before waiting for the projections.
+    const int pre = min(kKvStages - 1, ntiles);   // tiles loaded ahead of the loop
+    int loaded = 0;
+    while (loaded < pre && cs + (loaded + 1) * KT <= a.p0) load_tile(loaded++);
     asm volatile("griddepcontrol.wait;" ::: "memory");
 
     // 1. new K/V rows of this chunk -> cache (generic stores, then barrier)
     write_new_kv<__nv_bfloat16, NPL>(a, h, cs, ce);
     __syncthreads();
-    if (!early) load_tile(0);
+    while (loaded < pre) load_tile(loaded++);
 
     // 2. queries: m = r * G + gq, scaled into the log2 domain, bf16
     const float qscale = kLog2e * rsqrtf((float)HD);
@@ -268,142 +280,205 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const AttnArgs a) {
         }
     }
 
-    // 3. rounds of up to four m-tiles (one per warp) over the chunk's key tiles
-    for (int mt0 = 0; mt0 < mtiles; mt0 += kAttnWarps) {
-        const int mt = mt0 + warp;
-        const bool active = mt < mtiles;
-        if (mt0 > 0) load_tile(0);  // a new round streams the chunk again
-        uint32_t qf[HD / 16][4];
-        int rpos[2] = {-1, -1};
-        float o[NDT][4];
-        float mrow[2] = {-INFINITY, -INFINITY};
-        float lrow[2] = {0.f, 0.f};
+    // 3. rounds of up to two m-tiles.  In a round the four warps split every
+    //    64-key tile: warp w scores keys 16 w .. 16 w + 15 (Q K^T) and
+    //    accumulates head dims w HD/4 .. (w + 1) HD/4 of P V over all 64 keys.
+    //    Row maxima and row sums meet in shared memory and are combined in
+    //    warp order, so a row's arithmetic is the same for every R.
+    constexpr int WD = HD / kAttnWarps;   // head dims per warp
+    constexpr int WNT = WD / 8;           // n8 tiles of P V per warp
+    constexpr int PP = KT + 8;            // pitch of the probability tile
+    __shared__ __align__(16) __nv_bfloat16 Ps[2][16 * PP];
+    __shared__ float red_max[2][kAttnWarps][16];
+    __shared__ float red_sum[2][kAttnWarps][16];
+    for (int mt0 = 0; mt0 < mtiles; mt0 += 2) {
+        const int nm = min(2, mtiles - mt0);
+        if (mt0 > 0)   // a new round streams the chunk again
+            for (int j = 0; j < pre; ++j) load_tile(j);
+        uint32_t qf[2][HD / 16][4];
+        int rpos[2][2];
+        float o[2][WNT][4];
+        float mrow[2][2], lrow[2][2];
 #pragma unroll
-        for (int i = 0; i < NDT; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
+        for (int u = 0; u < 2; ++u)
+#pragma unroll
+            for (int hh = 0; hh < 2; ++hh) {
+                mrow[u][hh] = -INFINITY;
+                lrow[u][hh] = 0.f;
+                rpos[u][hh] = -1;
+            }
+#pragma unroll
+        for (int u = 0; u < 2; ++u)
+#pragma unroll
+            for (int i = 0; i < WNT; ++i) o[u][i][0] = o[u][i][1] = o[u][i][2] = o[u][i][3] = 0.f;
         bool qloaded = false;
 
         for (int ti = 0; ti < ntiles; ++ti) {
-            if (ti + 1 < ntiles) {
-                load_tile(ti + 1);
-                cp_async_wait<1>();
+            // tile ti + kKvStages - 1 goes into the slot tile ti - 1 used
+            if (ti + kKvStages - 1 < ntiles) {
+                load_tile(ti + kKvStages - 1);
+                cp_async_wait<kKvStages - 1>();
+            } else if (ti + 1 < ntiles) {
+                cp_async_wait<1>();   // tile ti + 1 may stay in flight
             } else {
                 cp_async_wait<0>();
             }
             __syncthreads();  // tile ti (and, first time, Qs) visible
-            if (active) {
-                if (!qloaded) {
+            if (!qloaded) {
+#pragma unroll
+                for (int u = 0; u < 2; ++u) {
+                    if (u >= nm) break;
+                    const int mt = mt0 + u;
 #pragma unroll
                     for (int ks = 0; ks < HD / 16; ++ks) {
                         const int mi = lane >> 3;
                         const int row = mt * 16 + (mi & 1) * 8 + (lane & 7);
                         const int col = ks * 16 + (mi >> 1) * 8;
-                        ldmatrix_x4(qf[ks], Qs + row * P + col);
+                        ldmatrix_x4(qf[u][ks], Qs + row * P + col);
                     }
 #pragma unroll
                     for (int hh = 0; hh < 2; ++hh) {
                         const int m = mt * 16 + g + 8 * hh;
-                        rpos[hh] = (m < M) ? a.p0 + m / G : -1;  // padding rows see no key
+                        rpos[u][hh] = (m < M) ? a.p0 + m / G : -1;  // padding rows see no key
                     }
-                    qloaded = true;
                 }
-                const __nv_bfloat16* Ks = KV + (size_t)(ti & 1) * 2 * KT * P;
-                const __nv_bfloat16* Vs = Ks + (size_t)KT * P;
-                const int kbase = cs + ti * KT;
+                qloaded = true;
+            }
+            const __nv_bfloat16* Ks = KV + (size_t)(ti % kKvStages) * 2 * KT * HD;
+            const __nv_bfloat16* Vs = Ks + (size_t)KT * HD;
+            const int kk = 16 * warp;               // this warp's keys in the tile
+            const int kbase = cs + ti * KT + kk;
+            // (a) scores of this warp's 16 keys, masked; row maxima to smem
+            float sc[2][2][4];
 #pragma unroll
-                for (int kk = 0; kk < KT; kk += 16) {
-                    float s[2][4];
+            for (int u = 0; u < 2; ++u) {
+                if (u >= nm) break;
 #pragma unroll
-                    for (int j = 0; j < 2; ++j) s[j][0] = s[j][1] = s[j][2] = s[j][3] = 0.f;
+                for (int j = 0; j < 2; ++j) sc[u][j][0] = sc[u][j][1] = sc[u][j][2] = sc[u][j][3] = 0.f;
 #pragma unroll
-                    for (int ks = 0; ks < HD / 16; ++ks) {
-                        uint32_t kb[4];
-                        const int mi = lane >> 3;
-                        const int krow = kk + (mi >> 1) * 8 + (lane & 7);
-                        const int kcol = ks * 16 + (mi & 1) * 8;
-                        ldmatrix_x4(kb, Ks + krow * P + kcol);
-                        mma_bf16(s[0], qf[ks][0], qf[ks][1], qf[ks][2], qf[ks][3], kb[0], kb[1]);
-                        mma_bf16(s[1], qf[ks][0], qf[ks][1], qf[ks][2], qf[ks][3], kb[2], kb[3]);
-                    }
-                    // causal / validity mask and online softmax (log2 domain)
+                for (int ks = 0; ks < HD / 16; ++ks) {
+                    uint32_t kb[4];
+                    const int mi = lane >> 3;
+                    const int krow = kk + (mi >> 1) * 8 + (lane & 7);
+                    const int kcol = ks * 16 + (mi & 1) * 8;
+                    ldmatrix_x4(kb, Ks + kv_off<HD>(krow, kcol));
+                    mma_bf16(sc[u][0], qf[u][ks][0], qf[u][ks][1], qf[u][ks][2], qf[u][ks][3], kb[0], kb[1]);
+                    mma_bf16(sc[u][1], qf[u][ks][0], qf[u][ks][1], qf[u][ks][2], qf[u][ks][3], kb[2], kb[3]);
+                }
 #pragma unroll
-                    for (int hh = 0; hh < 2; ++hh) {
-                        float tmax = -INFINITY;
+                for (int hh = 0; hh < 2; ++hh) {
+                    float tmax = -INFINITY;
+#pragma unroll
+                    for (int j = 0; j < 2; ++j)
+#pragma unroll
+                        for (int e = 0; e < 2; ++e) {
+                            const int key = kbase + j * 8 + 2 * t + e;
+                            float& v = sc[u][j][2 * hh + e];
+                            if (key > rpos[u][hh] || key >= ce) v = -INFINITY;
+                            tmax = fmaxf(tmax, v);
+                        }
+                    tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 1));
+                    tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 2));
+                    if (t == 0) red_max[u][warp][g + 8 * hh] = tmax;
+                }
+            }
+            __syncthreads();
+            // (b) the tile's row maximum, probabilities to smem, row sums to smem
+            float alpha[2][2];
+#pragma unroll
+            for (int u = 0; u < 2; ++u) {
+                if (u >= nm) break;
+#pragma unroll
+                for (int hh = 0; hh < 2; ++hh) {
+                    const int row = g + 8 * hh;
+                    const float tile_max = fmaxf(fmaxf(red_max[u][0][row], red_max[u][1][row]),
+                                                 fmaxf(red_max[u][2][row], red_max[u][3][row]));
+                    const float mnew = fmaxf(mrow[u][hh], tile_max);
+                    float psum = 0.f;
+                    if (mnew == -INFINITY) {
+                        alpha[u][hh] = 1.f;
+#pragma unroll
+                        for (int j = 0; j < 2; ++j) sc[u][j][2 * hh] = sc[u][j][2 * hh + 1] = 0.f;
+                    } else {
+                        alpha[u][hh] = exp2f(mrow[u][hh] - mnew);
 #pragma unroll
                         for (int j = 0; j < 2; ++j)
 #pragma unroll
                             for (int e = 0; e < 2; ++e) {
-                                const int key = kbase + kk + j * 8 + 2 * t + e;
-                                float& v = s[j][2 * hh + e];
-                                if (key > rpos[hh] || key >= ce) v = -INFINITY;
-                                tmax = fmaxf(tmax, v);
+                                float& v = sc[u][j][2 * hh + e];
+                                v = exp2f(v - mnew);
+                                psum += v;
                             }
-                        tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 1));
-                        tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 2));
-                        const float mnew = fmaxf(mrow[hh], tmax);
-                        float alpha, psum = 0.f;
-                        if (mnew == -INFINITY) {
-                            alpha = 1.f;
-#pragma unroll
-                            for (int j = 0; j < 2; ++j) s[j][2 * hh] = s[j][2 * hh + 1] = 0.f;
-                        } else {
-                            alpha = exp2f(mrow[hh] - mnew);
-#pragma unroll
-                            for (int j = 0; j < 2; ++j)
-#pragma unroll
-                                for (int e = 0; e < 2; ++e) {
-                                    float& v = s[j][2 * hh + e];
-                                    v = exp2f(v - mnew);
-                                    psum += v;
-                                }
-                        }
-                        mrow[hh] = mnew;
-                        lrow[hh] = lrow[hh] * alpha + psum;
-#pragma unroll
-                        for (int i = 0; i < NDT; ++i) {
-                            o[i][2 * hh] *= alpha;
-                            o[i][2 * hh + 1] *= alpha;
-                        }
                     }
-                    // O += P V
-                    const uint32_t pa0 = pack_bf16(s[0][0], s[0][1]);
-                    const uint32_t pa1 = pack_bf16(s[0][2], s[0][3]);
-                    const uint32_t pa2 = pack_bf16(s[1][0], s[1][1]);
-                    const uint32_t pa3 = pack_bf16(s[1][2], s[1][3]);
+                    mrow[u][hh] = mnew;
+                    psum += __shfl_xor_sync(0xffffffffu, psum, 1);
+                    psum += __shfl_xor_sync(0xffffffffu, psum, 2);
+                    if (t == 0) red_sum[u][warp][row] = psum;
 #pragma unroll
-                    for (int dp = 0; dp < NDT / 2; ++dp) {
+                    for (int j = 0; j < 2; ++j)
+                        *reinterpret_cast<uint32_t*>(&Ps[u][row * PP + kk + 8 * j + 2 * t]) =
+                            pack_bf16(sc[u][j][2 * hh], sc[u][j][2 * hh + 1]);
+                }
+            }
+            __syncthreads();
+            // (c) l and o rescaled; O += P V over the 64 keys for this warp's dims
+#pragma unroll
+            for (int u = 0; u < 2; ++u) {
+                if (u >= nm) break;
+#pragma unroll
+                for (int hh = 0; hh < 2; ++hh) {
+                    const int row = g + 8 * hh;
+                    const float tsum = ((red_sum[u][0][row] + red_sum[u][1][row]) + red_sum[u][2][row]) +
+                                       red_sum[u][3][row];
+                    lrow[u][hh] = lrow[u][hh] * alpha[u][hh] + tsum;
+#pragma unroll
+                    for (int i = 0; i < WNT; ++i) {
+                        o[u][i][2 * hh] *= alpha[u][hh];
+                        o[u][i][2 * hh + 1] *= alpha[u][hh];
+                    }
+                }
+#pragma unroll
+                for (int kq = 0; kq < KT / 16; ++kq) {
+                    uint32_t pa[4];
+                    {
+                        const int mi = lane >> 3;
+                        const int row = (mi & 1) * 8 + (lane & 7);
+                        const int col = kq * 16 + (mi >> 1) * 8;
+                        ldmatrix_x4(pa, &Ps[u][row * PP + col]);
+                    }
+#pragma unroll
+                    for (int dq = 0; dq < WNT / 2; ++dq) {
                         uint32_t vb[4];
                         const int mi = lane >> 3;
-                        const int vrow = kk + (mi & 1) * 8 + (lane & 7);
-                        const int vcol = dp * 16 + (mi >> 1) * 8;
-                        ldmatrix_x4_trans(vb, Vs + vrow * P + vcol);
-                        mma_bf16(o[2 * dp], pa0, pa1, pa2, pa3, vb[0], vb[1]);
-                        mma_bf16(o[2 * dp + 1], pa0, pa1, pa2, pa3, vb[2], vb[3]);
+                        const int vrow = kq * 16 + (mi & 1) * 8 + (lane & 7);
+                        const int vcol = warp * WD + dq * 16 + (mi >> 1) * 8;
+                        ldmatrix_x4_trans(vb, Vs + kv_off<HD>(vrow, vcol));
+                        mma_bf16(o[u][2 * dq], pa[0], pa[1], pa[2], pa[3], vb[0], vb[1]);
+                        mma_bf16(o[u][2 * dq + 1], pa[0], pa[1], pa[2], pa[3], vb[2], vb[3]);
                     }
                 }
             }
-            __syncthreads();  // everyone is done with tile ti before it is refilled
+            __syncthreads();  // everyone is done with tile ti (and Ps, red_*) before reuse
         }
-        if (!active) continue;
-        // full row sums of l across the quad, then this chunk's partials
+        // this chunk's partials: m and l by warp 0, each warp its dims of o
 #pragma unroll
-        for (int hh = 0; hh < 2; ++hh) {
-            lrow[hh] += __shfl_xor_sync(0xffffffffu, lrow[hh], 1);
-            lrow[hh] += __shfl_xor_sync(0xffffffffu, lrow[hh], 2);
-        }
+        for (int u = 0; u < 2; ++u) {
+            if (u >= nm) break;
 #pragma unroll
-        for (int hh = 0; hh < 2; ++hh) {
-            const int m = mt * 16 + g + 8 * hh;
-            if (m >= M) continue;
-            const int r = m / G, gq = m - r * G;
-            float* dst = a.part + (((size_t)r * a.hq + h * G + gq) * a.n_chunks_max + c) * (HD + kPartPad);
-            if (t == 0) {
-                dst[0] = mrow[hh];
-                dst[1] = lrow[hh];
-            }
+            for (int hh = 0; hh < 2; ++hh) {
+                const int m = (mt0 + u) * 16 + g + 8 * hh;
+                if (m >= M) continue;
+                const int r = m / G, gq = m - r * G;
+                float* dst = a.part + (((size_t)r * a.hq + h * G + gq) * a.n_chunks_max + c) * (HD + kPartPad);
+                if (warp == 0 && t == 0) {
+                    dst[0] = mrow[u][hh];
+                    dst[1] = lrow[u][hh];
+                }
 #pragma unroll
-            for (int i = 0; i < NDT; ++i) {
-                dst[kPartPad + i * 8 + 2 * t] = o[i][2 * hh];
-                dst[kPartPad + i * 8 + 2 * t + 1] = o[i][2 * hh + 1];
+                for (int i = 0; i < WNT; ++i) {
+                    dst[kPartPad + warp * WD + i * 8 + 2 * t] = o[u][i][2 * hh];
+                    dst[kPartPad + warp * WD + i * 8 + 2 * t + 1] = o[u][i][2 * hh + 1];
+                }
             }
         }
     }
@@ -544,7 +619,7 @@ __global__ void __launch_bounds__(128) attn_merge_kernel(const AttnArgs a) {
 // --------------------------------------------------------------- launchers
 static size_t attn_bf16_smem(int HD, int mpad) {
     const int P = HD + 8;
-    return sizeof(__nv_bfloat16) * ((size_t)mpad * P + 2 * 2 * (size_t)kKeyTile * P);
+    return sizeof(__nv_bfloat16) * ((size_t)mpad * P + (size_t)kKvStages * 2 * kKeyTile * HD);
 }
 
 cudaError_t launch_attention(int dtype, const AttnArgs& a, cudaStream_t s) {
