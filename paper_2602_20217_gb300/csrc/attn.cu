@@ -592,7 +592,8 @@ __global__ void __launch_bounds__(128) attn_merge_kernel(const AttnArgs a) {
     float o[PER];
 #pragma unroll
     for (int i = 0; i < PER; ++i) o[i] = 0.f;
-    for (int c = warp; c < nch; c += kAttnWarps) {
+#pragma unroll 8
+    for (int c = warp; c < nch; c += kAttnWarps) {   // unrolled: several chunks' loads in flight
         const float w = wsh[c];
         const float* src = base + (size_t)c * S + kPartPad + PER * lane;
         if constexpr (PER == 4) {

@@ -87,6 +87,18 @@ KS_DEV Phase decode(const ChainArgs& a, int k) {
     return p;
 }
 KS_DEV bool normed_input(int kind) { return kind == CH_QKV || kind == CH_GU || kind == CH_LM; }
+KS_DEV int stage_cols(int kind) { return kind == CH_GU ? 512 : 1024; }
+
+// Wavefront between phases: a stage of phase k reads columns kt * cols ..
+// of phase k - 1's output, so it waits only for the row groups that produce
+// them (block kt of phase k - 1), not for the whole phase.  Each finished row
+// group of phase k - 1 adds 1 to its block's counter.
+constexpr int kMaxBlocks = 64;
+KS_DEV int block_rowgroups(int n_out, int cols, int b) {   // row groups of block b
+    const int first = b * (cols / 16);
+    const int last = min((n_out + 15) / 16, (b + 1) * (cols / 16));
+    return last - first;
+}
 KS_DEV const CUtensorMap* amap_of(const ChainArgs& a, int kind) {
     return &a.amap[kind == CH_GU ? 1 : kind == CH_O ? 2 : kind == CH_DOWN ? 3 : 0];
 }
@@ -254,6 +266,7 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
     int* queue = a.counters;
     int* done = a.counters + kChainMaxPhases;
     int* exits = a.counters + 2 * kChainMaxPhases;
+    int* blocks = a.counters + 2 * kChainMaxPhases + 1;   // [phase][kMaxBlocks]
 
     if (tid == 0) {
         for (int i = 0; i < S; ++i) {
@@ -344,8 +357,8 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
     } else if (warp == kWarpA) {
         // ---------------------------------------------- activation loader
         grid_dependency_wait();   // the first phase's input comes from the previous kernel
-        int cur = -1;
-        bool ok = true;
+        int cur = -1, ready = 0;
+        bool scaled = false, ok = true;
         for (int t = 0;; ++t) {
             const int slot = t % S;
             // lane 0 waits; the shuffle broadcasts the outcome and orders the
@@ -364,12 +377,28 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
             const int kt = slot_kt[slot];
             const Phase P = decode(a, k);
             if (k != cur) {
+                cur = k;
+                ready = 0;      // blocks of phase k - 1 known to be complete
+                scaled = false;
+            }
+            if (k > 0 && kt >= ready) {
+                // wait for the block of phase k - 1 that this stage reads
+                const int n_prev = decode(a, k - 1).N;
                 bool dep = true;
-                if (lane == 0 && k > 0) dep = wait_at_least(&done[k - 1], decode(a, k - 1).n_items, kWaitLimitNs);
+                if (lane == 0)
+                    dep = wait_at_least(&blocks[(k - 1) * kMaxBlocks + kt],
+                                        block_rowgroups(n_prev, stage_cols(P.kind), kt), kWaitLimitNs);
                 if (!__shfl_sync(0xffffffffu, (int)dep, 0)) {
                     ok = false;
                     break;
                 }
+                fence_proxy_async_global();
+                if (kt == ready) ++ready;   // stages of an item come in order
+            }
+            // The 1/rms scale needs all of phase k - 1: ready when this item's
+            // last stage had its block (an item's stages cover every block).
+            if (!scaled && kt == P.tpi - 1) {
+                scaled = true;
                 if (normed_input(P.kind)) {
                     // 1 / rms of each row from the 16-feature partial sums of
                     // squares: lane l adds groups l, l + 32, ..., then a
@@ -384,9 +413,7 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
                 } else if (lane < kMaxRows) {
                     scale[k & 1][lane] = 1.f;
                 }
-                fence_proxy_async_global();
                 __syncwarp();
-                cur = k;
             }
             if (lane == 0) {
                 const int nb = (P.kind == CH_GU) ? 2 : 4;
@@ -521,6 +548,15 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
             if (lane == 0) mbar_arrive(&red_free[b]);   // partials read: the buffer is free
             epilogue<NT>(a, P, k, it, acc, accu, scale[k & 1], run_v, run_i);
             ++items_in_phase;
+            if (k + 1 < a.n_phases) {
+                // publish this row group to the next phase's stages that read it
+                fence_proxy_async_global();
+                __syncwarp();
+                if (lane == 0) {
+                    __threadfence();
+                    atomicAdd(&blocks[k * kMaxBlocks + (it * 16) / stage_cols(decode(a, k + 1).kind)], 1);
+                }
+            }
             if (last_item) {
                 // this CTA has no more items in the phase: publish them all
                 // with one release (the next phase reads them by TMA)
@@ -567,6 +603,7 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
             for (int k = 0; k < a.n_phases; ++k) {
                 queue[k] = 0;
                 done[k] = 0;
+                for (int b = 0; b < kMaxBlocks; ++b) blocks[k * kMaxBlocks + b] = 0;
             }
             *exits = 0;
             __threadfence();
@@ -576,7 +613,7 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
 
 }  // namespace
 
-size_t chain_counter_ints() { return 2 * (size_t)kChainMaxPhases + 1; }
+size_t chain_counter_ints() { return 2 * (size_t)kChainMaxPhases + 1 + (size_t)kChainMaxPhases * kMaxBlocks; }
 
 cudaError_t launch_chain(const ChainArgs& args, cudaStream_t s) {
     if (args.R < 1 || args.R > kMaxRows || args.n_phases < 1 || args.n_phases > kChainMaxPhases ||

@@ -101,6 +101,9 @@ static bool config_ok(const ks_config* c) {
     if (c->n_q_heads / c->n_kv_heads > 16) return false;
     if (c->head_dim != 64 && c->head_dim != 128) return false;
     if (c->d_ff < 8 || c->d_ff % 8) return false;
+    // the chain kernel's per-block counters: at most 64 blocks of a phase's
+    // output (512 columns for gate/up inputs, 1024 otherwise)
+    if (c->d_model > 64 * 512 || c->d_ff > 64 * 1024) return false;
     if (c->vocab < 1) return false;
     if (c->dtype != KS_DTYPE_F32 && c->dtype != KS_DTYPE_BF16) return false;
     if (c->max_seq < 2 || c->max_rows < 2 || c->max_rows > 16) return false;
