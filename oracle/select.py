@@ -11,6 +11,9 @@ Follows:
   w = round(t / Delta).
 * Sec. 3.3: each sublayer is a knapsack item; its latency is the weight and
   its similarity to the target's representation is the value.
+* Sec. 3.5 / Alg. 2 / Eq. 4: the TPT stage - candidate layer sets, acceptance
+  estimated on the history rows, grid search of Eq. 3 over candidates and
+  draft lengths (readings at the end of this file).
 
 Readings (listed in the design notes):
 * Item value.  The value of running sublayer i is the similarity the draft
@@ -191,3 +194,89 @@ def tpt(alpha: float, gamma: int, td: float, tt: float) -> float:
 def tpl(alpha: float, gamma: int, exit_layer: int, n_layers: int) -> float:
     """Eq. 2 (DEL's tokens per layer)."""
     return expected_tokens(alpha, gamma) / (gamma * exit_layer + n_layers)
+
+
+# ------------------------------------------------- TPT stage (NEXT row 1)
+# Alg. 2 selects (S*, gamma*) from a candidate set A of layer sets: the
+# knapsack optimum for each of several latency budgets (Sec. 3.3 / 3.5), an
+# acceptance estimate alpha_S per candidate from the history (Eq. 4), and a
+# grid search of Eq. 3 over A x [D].  Readings (listed in the design notes):
+# * A: the optimal masks for the K budgets floor(sum_w * (j + 1) / K), j < K;
+# * the draft's final hidden state on a history row is estimated to first
+#   order from the recorded sublayer outputs: the target's X^(2L) minus the
+#   contribution X^(i) - X^(i-1) of every skipped sublayer i (the paper's
+#   propagated DP state of Alg. 1 is not built);
+# * a prediction is the argmax of the LM head on the final-normalised state,
+#   and the target tokens are those of the full layer set on the same rows;
+# * Eq. 1 is summed term by term with alpha^i formed by repeated products.
+def frontier_budgets(total_w: int, k: int) -> list:
+    """Candidate budgets floor(total_w * (j + 1) / K) for j = 0..K-1."""
+    return [(int(total_w) * (j + 1)) // int(k) for j in range(int(k))]
+
+
+def frontier(weights, values, k: int):
+    """The candidate set A: one optimal knapsack mask per candidate budget.
+    Returns (list of uint8 masks, list of budgets)."""
+    budgets = frontier_budgets(int(np.sum(weights)), k)
+    return [knapsack(weights, values, c)[0] for c in budgets], budgets
+
+
+def draft_states(hist: np.ndarray, mask) -> np.ndarray:
+    """First-order final state of f^(S) on the history rows: X^(2L) minus the
+    recorded contribution of each skipped sublayer.  hist is [2L+1, r, d]."""
+    hist = np.asarray(hist, np.float64)
+    h = hist[-1].copy()
+    for i in range(1, hist.shape[0]):
+        if not mask[i - 1]:
+            h -= hist[i] - hist[i - 1]
+    return h
+
+
+def lm_argmax(states: np.ndarray, lm_head: np.ndarray, final_gain: np.ndarray, eps: float) -> np.ndarray:
+    """Token predicted from each row: final RMSNorm, LM head, argmax (ties to
+    the lowest id)."""
+    x = np.asarray(states, np.float64)
+    x = x / np.sqrt(np.mean(x * x, axis=-1, keepdims=True) + eps) * np.asarray(final_gain, np.float64)
+    return np.argmax(x @ np.asarray(lm_head, np.float64).T, axis=-1).astype(np.int64)
+
+
+def alpha_hat(pred, target) -> float:
+    """Eq. 4: the fraction of history rows on which the draft's prediction
+    equals the target's token."""
+    pred = np.asarray(pred)
+    return float(np.count_nonzero(pred == np.asarray(target))) / float(len(pred))
+
+
+def expected_tokens_iter(alpha: float, gamma: int) -> float:
+    """Eq. 1 as a sum, alpha^i by repeated products (the order the device uses)."""
+    e, p = 1.0, 1.0
+    for _ in range(int(gamma)):
+        p = p * alpha
+        e = e + p
+    return e
+
+
+def select_tpt(masks, alphas, n_layers: int, max_gamma: int, ta: float = None, tm: float = None, units=None):
+    """Alg. 2's grid search: candidates in order, gamma = 1..D ascending, a pair
+    replaces the best only when its TPT (Eq. 3) is strictly larger.  Latencies
+    are t_Attn / t_MLP, or explicit per-sublayer units.
+    Returns (candidate index, gamma, tpt)."""
+    best = (-1, 0, 0.0)
+    if units is not None:
+        units = [float(u) for u in units]
+        tt = float(sum(units))
+    else:
+        tt = t_target(n_layers, ta, tm)
+    for j, (m, a) in enumerate(zip(masks, alphas)):
+        if units is not None:
+            td = 0.0
+            for i, u in enumerate(units):
+                if m[i]:
+                    td = td + u
+        else:
+            td = t_draft(m, ta, tm)
+        for g in range(1, int(max_gamma) + 1):
+            v = expected_tokens_iter(a, g) / (g * td + tt)
+            if v > best[2]:
+                best = (j, g, v)
+    return best

@@ -13,6 +13,12 @@ What pins what:
 * Eq. 1: closed form (1 - a^(g+1)) / (1 - a), limits a -> 0 and a -> 1, and a
   Monte-Carlo truncated-geometric simulation.
 * Eq. 3: TPT reduces to TPL (Eq. 2) when t_Attn = t_MLP (Sec. 3.2).
+* TPT stage (Alg. 2): the estimated draft states telescope to X^(2L) (full
+  set) and X^(0) (empty set) and equal the forward sum of kept
+  contributions; each frontier mask is the brute-force optimum of its
+  budget; Eq. 4 on the full set is 1; the LM-head argmax against a row-by-row
+  loop; the grid search against brute force, alpha = 0 (gamma = 1) and
+  alpha = 1 with a cheaper draft (gamma = D).
 """
 import json
 import os
@@ -195,3 +201,80 @@ def test_tpt_reduces_to_tpl_with_equal_latencies():
 def test_t_draft_counts_attn_and_mlp():
     mask = np.array([1, 0, 1, 1, 0, 1])   # sublayers 1,3 (Attn) and 4,6 (MLP) run
     assert S.t_draft(mask, 10.0, 1.0) == 2 * 10.0 + 2 * 1.0
+
+
+# ------------------------------------------------------ TPT stage (NEXT-1)
+def _history(seed=0, L=3, r=5, d=16):
+    rng = np.random.default_rng(seed)
+    return np.cumsum(rng.standard_normal((2 * L + 1, r, d)), axis=0)
+
+
+def test_draft_states_telescope_to_the_endpoints():
+    hist = _history()
+    n = hist.shape[0] - 1
+    assert np.allclose(S.draft_states(hist, np.ones(n, np.uint8)), hist[-1], atol=1e-12)
+    assert np.allclose(S.draft_states(hist, np.zeros(n, np.uint8)), hist[0], atol=1e-12)
+    mask = np.array([1, 0, 0, 1, 1, 0], np.uint8)
+    # the same state built forwards: X^(0) plus the kept contributions
+    fwd = hist[0] + sum(hist[i] - hist[i - 1] for i in range(1, n + 1) if mask[i - 1])
+    assert np.allclose(S.draft_states(hist, mask), fwd, atol=1e-12)
+
+
+def test_frontier_is_the_knapsack_optimum_per_budget():
+    rng = np.random.default_rng(3)
+    w = rng.integers(1, 5, 10)
+    q = rng.integers(0, 1000, 10)
+    masks, budgets = S.frontier(w, q, 6)
+    assert budgets[-1] == int(w.sum()) and budgets == sorted(budgets)
+    vals = []
+    for m, b in zip(masks, budgets):
+        bm, bv = S.knapsack_brute(w, q, b)
+        assert np.array_equal(m, bm)
+        vals.append(int(m.astype(np.int64) @ q))
+    assert vals == sorted(vals)   # a larger budget never lowers the objective
+
+
+def test_alpha_hat_full_set_is_one_and_lm_argmax_matches_definition():
+    rng = np.random.default_rng(1)
+    hist = _history(1, L=2, r=7, d=12)
+    W = rng.standard_normal((30, 12))
+    g = rng.uniform(0.5, 1.5, 12)
+    target = S.lm_argmax(hist[-1], W, g, 1e-5)
+    full = S.lm_argmax(S.draft_states(hist, np.ones(4, np.uint8)), W, g, 1e-5)
+    assert S.alpha_hat(full, target) == 1.0
+    # argmax written out row by row
+    for i in range(7):
+        x = hist[-1][i]
+        y = x / np.sqrt(np.mean(x * x) + 1e-5) * g
+        assert target[i] == int(np.argmax([W[v] @ y for v in range(30)]))
+    assert S.alpha_hat([1, 2, 3, 4], [1, 0, 3, 0]) == 0.5
+
+
+def test_expected_tokens_iter_matches_closed_form():
+    for a in (0.0, 0.3, 0.9, 1.0):
+        for g in range(1, 11):
+            assert S.expected_tokens_iter(a, g) == pytest.approx(S.expected_tokens(a, g), rel=1e-14)
+
+
+def test_select_tpt_grid_search_special_cases():
+    masks = [np.array([0, 1, 0, 1], np.uint8), np.array([1, 1, 0, 1], np.uint8), np.ones(4, np.uint8)]
+    ta, tm = 2.0, 3.0
+    # brute force over the same grid
+    alphas = [0.4, 0.7, 1.0]
+    j, g, v = S.select_tpt(masks, alphas, 2, 10, ta=ta, tm=tm)
+    grid = [(S.tpt(a, gg, S.t_draft(m, ta, tm), S.t_target(2, ta, tm)), jj, gg)
+            for jj, (m, a) in enumerate(zip(masks, alphas)) for gg in range(1, 11)]
+    best = max(grid, key=lambda x: x[0])
+    assert (j, g) == (best[1], best[2]) and v == pytest.approx(best[0], rel=1e-12)
+    # alpha = 0 everywhere: one draft token is the least waste
+    assert S.select_tpt(masks, [0.0] * 3, 2, 10, ta=ta, tm=tm)[1] == 1
+    # alpha = 1 with a draft cheaper than the target: TPT grows with gamma
+    j1, g1, _ = S.select_tpt(masks[:1], [1.0], 2, 10, ta=ta, tm=tm)
+    assert (j1, g1) == (0, 10)
+    # explicit units act as latencies
+    u = [1, 2, 1, 2]
+    ju, gu, vu = S.select_tpt(masks, alphas, 2, 4, units=u)
+    gridu = [(S.expected_tokens(a, gg) / (gg * float(np.dot(m, u)) + 6.0), jj, gg)
+             for jj, (m, a) in enumerate(zip(masks, alphas)) for gg in range(1, 5)]
+    bu = max(gridu, key=lambda x: x[0])
+    assert (ju, gu) == (bu[1], bu[2])
