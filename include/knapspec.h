@@ -236,16 +236,46 @@ ks_status ks_select_mask_static(const ks_latency* lat, const float* sims, int64_
                                 int32_t n_sublayers, int32_t budget_units, uint8_t* mask_out,
                                 double* objective_out, int32_t* weights_out, void* stream);
 
+/* The TPT stage of the layer selection (Sec. 3.5, Alg. 2, Eqs. 1, 3, 4), on
+ * the model's history (the same rows as ks_history_similarities):
+ *  1. candidate set A: with the values of a4 and the weights of `lat` (as in
+ *     ks_select_mask), the knapsack optimum for each of n_candidates budgets
+ *     floor(sum_i w_i (j + 1) / n_candidates), j = 0 .. n_candidates - 1;
+ *  2. acceptance of each candidate on the r history rows (Eq. 4): the
+ *     draft's final state on a row is taken to first order as the target's
+ *     X^(2L) minus the recorded contribution X^(i) - X^(i-1) of every skipped
+ *     sublayer i; its prediction (final RMSNorm, LM head, argmax, ties to the
+ *     lowest id) is compared with the full layer set's on the same row;
+ *  3. grid search of Eq. 3 over A x {1 .. max_gamma}: expected tokens (Eq. 1)
+ *     over gamma t_Draft(S) + t_Target, with t_Attn(n) and t_MLP of the
+ *     latency model (kind 0, n = the committed length) or the units as times
+ *     (kind 1); candidates in order, gamma ascending, strictly larger wins.
+ * n_candidates: 1 .. KS_TPT_MAX_CANDIDATES; max_gamma: 1 .. max_rows - 1.
+ * Outputs (host): mask_out[2L] (the chosen candidate), *gamma_out, *tpt_out
+ * (in tokens per unit of the latency's time), and, unless NULL,
+ * alphas_out[n_candidates] and candidates_out[n_candidates][2L].  Uses the
+ * model's pass buffers but no decoding state changes.  Waits for the stream.
+ * KS_ERR_STATE before a prefill. */
+#define KS_TPT_MAX_CANDIDATES 16
+ks_status ks_select_tpt(ks_model* m, const ks_latency* lat, int32_t n_candidates, int32_t max_gamma,
+                        uint8_t* mask_out, int32_t* gamma_out, double* tpt_out, double* alphas_out,
+                        uint8_t* candidates_out);
+
 /* ------------------------------------------------- full speculative loop */
 
 typedef struct {
-    int32_t gamma;           /* draft length per step (1 <= gamma < max_rows)              */
-    int32_t policy;          /* 0 fixed mask, 1 knapsack re-solved every resolve_every steps */
+    int32_t gamma;           /* draft length per step (1 <= gamma < max_rows); policy 2: until
+                                the first selection                                         */
+    int32_t policy;          /* 0 fixed mask; 1 knapsack re-solved every resolve_every steps;
+                                2 TPT stage (ks_select_tpt) every resolve_every steps, which
+                                also sets gamma                                             */
     const uint8_t* mask;     /* host uint8[2L]: the mask for policy 0                      */
-    ks_latency latency;      /* policy 1                                                   */
+    ks_latency latency;      /* policies 1 and 2                                            */
     double budget_frac;      /* policy 1: budget = floor(budget_frac * sum_i w_i)          */
-    int32_t resolve_every;   /* policy 1: optimisation interval T in verify steps (>= 1)   */
+    int32_t resolve_every;   /* policies 1, 2: optimisation interval T in verify steps (>= 1) */
     int32_t max_steps;       /* stop after this many verify steps (0: no limit)             */
+    int32_t tpt_candidates;  /* policy 2: n_candidates of ks_select_tpt                     */
+    int32_t tpt_max_gamma;   /* policy 2: max_gamma of ks_select_tpt                        */
 } ks_spec_params;
 
 typedef struct {

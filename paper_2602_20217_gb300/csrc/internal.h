@@ -6,6 +6,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include "../../include/knapspec.h"
+
 namespace ks {
 
 // ------------------------------------------------------------------ GEMV
@@ -127,6 +129,16 @@ int attn_num_chunks(int n_keys);
 constexpr int kSsGroup = 16;    // features per sum-of-squares partial (= rows of a bf16 GEMV work item)
 
 // ---------------------------------------------------------------- select
+size_t select_scratch_bytes(int n_items, int cap);
+// Knapsack of a5 (optionally also the frontier of the TPT stage).
+cudaError_t launch_select(const ks_latency* lat, const float* sims, int64_t n, int n_items, int budget,
+                          double budget_frac, uint8_t* mask, double* objective, int32_t* weights,
+                          int32_t* budget_out, void* scratch, int cap, cudaStream_t s, int n_frontier = 0,
+                          uint8_t* frontier = nullptr);
+// TPT stage after the frontier: Eq. 4 acceptance per candidate and Eq. 3 grid.
+cudaError_t launch_tpt(const ks_latency* lat, int64_t n, int n_items, int n_layers, int K, int r, int D,
+                       const uint8_t* frontier, const int32_t* tokens, uint8_t* mask_out, int32_t* info,
+                       double* out, cudaStream_t s);
 cudaError_t launch_cosine(const void* X, const void* Y, int dtype, int64_t n_pairs, int rows,
                           int d, int64_t pair_stride, const int32_t* row_index, float* out,
                           cudaStream_t s);

@@ -15,6 +15,7 @@
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
+#include <algorithm>
 #include <cstring>
 #include <vector>
 
@@ -29,10 +30,6 @@ void set_error(const char* fmt, ...) {
     va_end(ap);
 }
 
-size_t select_scratch_bytes(int n_items, int cap);
-cudaError_t launch_select(const ks_latency* lat, const float* sims, int64_t n, int n_items, int budget,
-                          double budget_frac, uint8_t* mask, double* objective, int32_t* weights,
-                          int32_t* budget_out, void* scratch, int cap, cudaStream_t s);
 
 constexpr int kSelectCap = 65535;
 constexpr int kKlasses = 10;
@@ -81,12 +78,45 @@ __global__ void accept_kernel(int32_t* rows, const int32_t* z, int gamma, int32_
     rows[0] = z[a];
 }
 
+// TPT stage, Eq. 4 inputs: row b of a batch is overall row q = row0 + b, i.e.
+// candidate j = q / r (j == K: the full layer set) on history row i = q % r.
+// Its draft state is X^(2L) minus X^(s) - X^(s-1) for every sublayer s the
+// candidate skips, in order s = 1 .. 2L; written as the LM head's input: the
+// fp32 residual, its bf16 x * final gain, and the 16-feature sums of squares.
+template <typename WT>
+__global__ void __launch_bounds__(256) tpt_states_kernel(const float* hist, long long plane, const int32_t* hidx,
+                                                         int r, int row0, int nsub, const uint8_t* masks, int K,
+                                                         int d, const WT* gain, float* x, float* ss,
+                                                         __nv_bfloat16* xg) {
+    const int b = blockIdx.x;
+    const int q = row0 + b;
+    const int j = q / r, i = q - j * r;
+    const uint8_t* mask = (j < K) ? masks + (size_t)j * nsub : nullptr;
+    const int k = blockIdx.y * 256 + threadIdx.x;
+    float h = 0.f;
+    if (k < d) {
+        const float* base = hist + (size_t)hidx[i] * d + k;
+        h = base[(size_t)nsub * plane];
+        if (mask)
+            for (int sl = 1; sl <= nsub; ++sl)
+                if (!mask[sl - 1]) h -= base[(size_t)sl * plane] - base[(size_t)(sl - 1) * plane];
+        x[(size_t)b * d + k] = h;
+        if (xg) xg[(size_t)b * d + k] = __float2bfloat16_rn(h * to_float(gain[k]));
+    }
+    float sq = h * h;   // lanes 0-15 and 16-31 of each warp form one 16-feature group
+#pragma unroll
+    for (int o = 8; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
+    const int lane = threadIdx.x & 31;
+    if ((lane & 15) == 0 && k < d) ss[(k / kSsGroup) * 16 + b] = sq;
+}
+
 // ------------------------------------------------------------------ helpers
 static size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
 struct Layout {
     size_t kv, rope, x, ss, xg, qkv, attn_out, act, attn_part, gemv_part, counters, logits, amax_val,
-        amax_idx, tok, hist, hist_snap, hist_idx, sims, mask, obj, wts, select, chain_ctr, best, total;
+        amax_idx, tok, hist, hist_snap, hist_idx, sims, mask, obj, wts, select, chain_ctr, best, tpt_masks,
+        tpt_tok, tpt_info, tpt_out, total;
     int n_chunks_max;
     size_t gemv_part_floats;
     int counters_n;
@@ -167,6 +197,12 @@ static Layout make_layout(const ks_config* c) {
     // bf16: two sets of chain counters
     L.chain_ctr = take(sizeof(int) * 2 * chain_counter_ints());
     L.best = take(sizeof(unsigned long long) * 16);
+    // TPT stage: candidate masks, predicted tokens of every (candidate + full
+    // set) x history row, the choice and its figures
+    L.tpt_masks = take((size_t)KS_TPT_MAX_CANDIDATES * nsub);
+    L.tpt_tok = take(sizeof(int32_t) * (KS_TPT_MAX_CANDIDATES + 1) * (size_t)L.hist_slots * R);
+    L.tpt_info = take(sizeof(int32_t) * 4);
+    L.tpt_out = take(sizeof(double) * (KS_TPT_MAX_CANDIDATES + 1));
     L.total = off;
     return L;
 }
@@ -205,6 +241,10 @@ struct ks_model {
     ChainArgs* chain = nullptr;  // bf16: parameter block of the chain launches (host)
     int* chain_ctr;           // two counter sets, alternating between chain launches
     unsigned long long* best; // LM head argmax keys of the chain kernel
+    uint8_t* tpt_masks;       // TPT stage buffers
+    int32_t* tpt_tok;
+    int32_t* tpt_info;
+    double* tpt_out;
     int chain_parity = 0;
     double* obj_dev;
     int* wts_dev;
@@ -634,6 +674,10 @@ ks_status ks_model_create(const ks_config* cfg, const ks_weights* w, void* works
     m->mask_dev = reinterpret_cast<uint8_t*>(b + lay.mask);
     m->chain_ctr = reinterpret_cast<int*>(b + lay.chain_ctr);
     m->best = reinterpret_cast<unsigned long long*>(b + lay.best);
+    m->tpt_masks = reinterpret_cast<uint8_t*>(b + lay.tpt_masks);
+    m->tpt_tok = reinterpret_cast<int32_t*>(b + lay.tpt_tok);
+    m->tpt_info = reinterpret_cast<int32_t*>(b + lay.tpt_info);
+    m->tpt_out = reinterpret_cast<double*>(b + lay.tpt_out);
     m->obj_dev = reinterpret_cast<double*>(b + lay.obj);
     m->wts_dev = reinterpret_cast<int*>(b + lay.wts);
     m->select = b + lay.select;
@@ -962,19 +1006,106 @@ static int history_rows(ks_model* m, int32_t* idx) {
     return r;
 }
 
-ks_status ks_history_similarities(ks_model* m, float* sims, int32_t* rows_used) {
-    if (!m || !sims) {
-        set_error("ks_history_similarities: null argument");
-        return KS_ERR_INVALID_ARG;
+// LM head + argmax of R rows whose input (x, xg, ss) is already in place.
+static ks_status lm_head_rows(ks_model* m, int R, int32_t* tokens) {
+    const ks_config& c = m->cfg;
+    const int d = c.d_model, L = c.n_layers;
+    cudaStream_t s = m->stream;
+    if (m->dtype == KS_DTYPE_BF16) {
+        if (!m->chain) m->chain = new ChainArgs();
+        ChainArgs& ca = *m->chain;
+        ca.amap[0] = m->map_xg[R - 1];
+        ca.amap[1] = m->map_xg2[R - 1];
+        ca.amap[2] = m->map_attn_out[R - 1];
+        ca.amap[3] = m->map_act[R - 1];
+        ca.R = R;
+        ca.n_layers = L; ca.d = d; ca.F = c.d_ff; ca.hqd = c.n_q_heads * c.head_dim;
+        ca.nqkv = (c.n_q_heads + 2 * c.n_kv_heads) * c.head_dim; ca.vocab = c.vocab;
+        ca.eps = c.rms_eps;
+        ca.x = m->x; ca.ss = m->ss; ca.xg = m->xg; ca.qkv = m->qkv;
+        ca.act = reinterpret_cast<__nv_bfloat16*>(m->act);
+        ca.logits = m->logits; ca.best = m->best; ca.tokens = tokens;
+        ca.capture = nullptr;
+        ca.err = m->err;
+        ca.n_phases = 1;
+        ca.code[0] = (uint16_t)(4 * L);
+        ca.gain[0] = nullptr;
+        ca.wmap[0] = m->map_lm;
+        ca.counters = m->chain_ctr + (size_t)m->chain_parity * chain_counter_ints();
+        m->chain_parity ^= 1;
+        return launch(m, K_LMHEAD, [&] { return launch_chain(ca, s); }, "tpt lm-head",
+                      2.0 * c.vocab * (double)d);
     }
-    if (!m->have_seq) {
-        set_error("ks_history_similarities: no sequence");
-        return KS_ERR_STATE;
+    GemvArgs g{};
+    g.W = m->lm_head;
+    g.dtype = m->dtype;
+    g.N = c.vocab;
+    g.K = d;
+    g.R = R;
+    g.partial = m->gemv_part;
+    g.counters = m->counters;
+    g.err = m->err;
+    g.ss_in = m->ss;
+    g.ss_groups = (d + kSsGroup - 1) / kSsGroup;
+    g.eps = c.rms_eps;
+    g.in = m->x;
+    g.in_ld = d;
+    g.norm_gain = m->final_norm;
+    g.logits = m->logits;
+    g.logits_ld = c.vocab;
+    g.amax_val = m->amax_val;
+    g.amax_idx = m->amax_idx;
+    g.tokens = tokens;
+    gemv_plan(g, EPI_LMHEAD);
+    return launch(m, K_LMHEAD, [&] { return launch_gemv(m->dtype, EPI_LMHEAD, g, s); }, "tpt lm-head");
+}
+
+static ks_status history_sims(ks_model* m, int* rows_out);
+
+// The TPT stage on the device (results stay in tpt_* and mask_dev).
+static ks_status tpt_stage(ks_model* m, const ks_latency* lat, int K, int D, int* rows_out) {
+    const ks_config& c = m->cfg;
+    const int nsub = m->nsub, d = c.d_model;
+    int r = 0;
+    KS_TRY(history_sims(m, &r));
+    // frontier: the knapsack over the whole weight sum, backtracked at K budgets
+    KS_TRY(launch(m, K_ACCEPT, [&] {
+        return launch_select(lat, m->sims, m->p, nsub, 0, 1.0, m->mask_dev, m->obj_dev, m->wts_dev,
+                             m->wts_dev + nsub, m->select, kSelectCap, m->stream, K, m->tpt_masks);
+    }, "tpt frontier"));
+    // predictions of every candidate (and of the full set) on every history row
+    const int total = (K + 1) * r;
+    const int64_t plane = (int64_t)m->lay.hist_slots * c.max_rows * d;
+    const bool bf = m->dtype == KS_DTYPE_BF16;
+    for (int row0 = 0; row0 < total; row0 += c.max_rows) {
+        const int B = std::min(c.max_rows, total - row0);
+        KS_TRY(launch(m, K_EMBED, [&]() -> cudaError_t {
+            if (bf)
+                tpt_states_kernel<__nv_bfloat16><<<dim3(B, (d + 255) / 256), 256, 0, m->stream>>>(
+                    hist_plane(m, 0), plane, m->hist_idx, r, row0, nsub, m->tpt_masks, K, d,
+                    reinterpret_cast<const __nv_bfloat16*>(m->final_norm), m->x, m->ss, m->xg);
+            else
+                tpt_states_kernel<float><<<dim3(B, (d + 255) / 256), 256, 0, m->stream>>>(
+                    hist_plane(m, 0), plane, m->hist_idx, r, row0, nsub, m->tpt_masks, K, d,
+                    reinterpret_cast<const float*>(m->final_norm), m->x, m->ss, nullptr);
+            return cudaGetLastError();
+        }, "tpt states"));
+        KS_TRY(lm_head_rows(m, B, m->tpt_tok + row0));
     }
+    KS_TRY(launch(m, K_ACCEPT, [&] {
+        return launch_tpt(lat, m->p, nsub, c.n_layers, K, r, D, m->tpt_masks, m->tpt_tok, m->mask_dev,
+                          m->tpt_info, m->tpt_out, m->stream);
+    }, "tpt grid"));
+    if (rows_out) *rows_out = r;
+    return KS_OK;
+}
+
+// a4 on the history rows (their indices uploaded to hist_idx) into sims.
+static ks_status history_cosines(ks_model* m, float* sims, int* rows_out) {
     int32_t* hidx = m->h_buf + m->cfg.max_seq + 4 * m->cfg.max_rows + 16;
     const int r = history_rows(m, hidx);
     if (r < 1) {
-        set_error("ks_history_similarities: empty history");
+        set_error("history similarities: empty history");
         return KS_ERR_STATE;
     }
     KS_CUDA(cudaMemcpyAsync(m->hist_idx, hidx, sizeof(int32_t) * r, cudaMemcpyHostToDevice, m->stream),
@@ -986,7 +1117,70 @@ ks_status ks_history_similarities(ks_model* m, float* sims, int32_t* rows_used) 
                                   m->hist_idx, sims, m->stream);
     if (e != cudaSuccess) return cuda_fail(e, "history cosine");
     m->launches++;
+    if (rows_out) *rows_out = r;
+    return KS_OK;
+}
+
+static ks_status history_sims(ks_model* m, int* rows_out) { return history_cosines(m, m->sims, rows_out); }
+
+ks_status ks_history_similarities(ks_model* m, float* sims, int32_t* rows_used) {
+    if (!m || !sims) {
+        set_error("ks_history_similarities: null argument");
+        return KS_ERR_INVALID_ARG;
+    }
+    if (!m->have_seq) {
+        set_error("ks_history_similarities: no sequence");
+        return KS_ERR_STATE;
+    }
+    int r = 0;
+    KS_TRY(history_cosines(m, sims, &r));
     if (rows_used) *rows_used = r;
+    return KS_OK;
+}
+
+static bool latency_ok(const ks_latency& lat, int nsub) {
+    bool ok = lat.kind == 0 ? (lat.c1 > 0 && lat.c2 >= 0 && lat.c3 >= 0 && std::isfinite(lat.c1) &&
+                               std::isfinite(lat.c2) && std::isfinite(lat.c3))
+                            : (lat.kind == 1 && lat.units);
+    if (ok && lat.kind == 1)
+        for (int i = 0; i < nsub; ++i) ok = ok && lat.units[i] >= 1 && lat.units[i] <= 65535;
+    return ok;
+}
+
+ks_status ks_select_tpt(ks_model* m, const ks_latency* lat, int32_t n_candidates, int32_t max_gamma,
+                        uint8_t* mask_out, int32_t* gamma_out, double* tpt_out, double* alphas_out,
+                        uint8_t* candidates_out) {
+    if (!m || !lat || !mask_out || !gamma_out || !tpt_out) {
+        set_error("ks_select_tpt: null argument");
+        return KS_ERR_INVALID_ARG;
+    }
+    if (n_candidates < 1 || n_candidates > KS_TPT_MAX_CANDIDATES || max_gamma < 1 ||
+        max_gamma >= m->cfg.max_rows || !latency_ok(*lat, m->nsub)) {
+        set_error("ks_select_tpt: bad argument");
+        return KS_ERR_INVALID_ARG;
+    }
+    if (!m->have_seq) {
+        set_error("ks_select_tpt: no sequence (call ks_prefill first)");
+        return KS_ERR_STATE;
+    }
+    KS_TRY(tpt_stage(m, lat, n_candidates, max_gamma, nullptr));
+    const int nsub = m->nsub;
+    std::vector<double> out(1 + n_candidates);
+    int32_t info[2] = {0, 0};
+    KS_CUDA(cudaMemcpyAsync(mask_out, m->mask_dev, nsub, cudaMemcpyDeviceToHost, m->stream), "tpt download");
+    KS_CUDA(cudaMemcpyAsync(info, m->tpt_info, sizeof(info), cudaMemcpyDeviceToHost, m->stream), "tpt download");
+    KS_CUDA(cudaMemcpyAsync(out.data(), m->tpt_out, sizeof(double) * out.size(), cudaMemcpyDeviceToHost, m->stream),
+            "tpt download");
+    if (candidates_out)
+        KS_CUDA(cudaMemcpyAsync(candidates_out, m->tpt_masks, (size_t)n_candidates * nsub, cudaMemcpyDeviceToHost,
+                                m->stream),
+                "tpt download");
+    m->d2h += nsub + sizeof(info) + sizeof(double) * out.size() + (candidates_out ? n_candidates * nsub : 0);
+    KS_TRY(sync(m, "ks_select_tpt"));
+    *gamma_out = info[1];
+    *tpt_out = out[0];
+    if (alphas_out)
+        for (int j = 0; j < n_candidates; ++j) alphas_out[j] = out[1 + j];
     return KS_OK;
 }
 
@@ -1001,21 +1195,18 @@ ks_status ks_generate_speculative(ks_model* m, const ks_spec_params* prm, int32_
         return KS_ERR_STATE;
     }
     const int nsub = m->nsub;
-    if (prm->gamma < 1 || prm->gamma >= m->cfg.max_rows || (prm->policy != 0 && prm->policy != 1) ||
+    if (prm->gamma < 1 || prm->gamma >= m->cfg.max_rows || prm->policy < 0 || prm->policy > 2 ||
         (prm->policy == 0 && !prm->mask) ||
-        (prm->policy == 1 && (prm->resolve_every < 1 || !(prm->budget_frac >= 0.0) || prm->budget_frac > 1.0))) {
+        (prm->policy == 1 && (prm->resolve_every < 1 || !(prm->budget_frac >= 0.0) || prm->budget_frac > 1.0)) ||
+        (prm->policy == 2 && (prm->resolve_every < 1 || prm->tpt_candidates < 1 ||
+                              prm->tpt_candidates > KS_TPT_MAX_CANDIDATES || prm->tpt_max_gamma < 1 ||
+                              prm->tpt_max_gamma >= m->cfg.max_rows))) {
         set_error("ks_generate_speculative: bad parameters");
         return KS_ERR_INVALID_ARG;
     }
-    if (prm->policy == 1) {
-        const ks_latency& lat = prm->latency;
-        bool ok = lat.kind == 0 ? (lat.c1 > 0 && lat.c2 >= 0 && lat.c3 >= 0) : (lat.kind == 1 && lat.units);
-        if (ok && lat.kind == 1)
-            for (int i = 0; i < nsub; ++i) ok = ok && lat.units[i] >= 1 && lat.units[i] <= 65535;
-        if (!ok) {
-            set_error("ks_generate_speculative: bad latency model");
-            return KS_ERR_INVALID_ARG;
-        }
+    if (prm->policy != 0 && !latency_ok(prm->latency, nsub)) {
+        set_error("ks_generate_speculative: bad latency model");
+        return KS_ERR_INVALID_ARG;
     }
     ks_spec_stats st{};
     std::vector<uint8_t> mask(nsub, 1);
@@ -1023,7 +1214,23 @@ ks_status ks_generate_speculative(ks_model* m, const ks_spec_params* prm, int32_
     int n = 0;
     out[n++] = m->pending;
     std::vector<int32_t> toks(m->cfg.max_rows + 1);
+    int gamma = prm->gamma;
     while (n < n_tokens && (prm->max_steps <= 0 || st.steps < prm->max_steps)) {
+        if (prm->policy == 2 && st.steps % prm->resolve_every == 0) {
+            // TPT stage: the next mask and draft length
+            KS_TRY(tpt_stage(m, &prm->latency, prm->tpt_candidates, prm->tpt_max_gamma, nullptr));
+            uint8_t* hm = reinterpret_cast<uint8_t*>(m->h_buf + m->cfg.max_seq + 4 * m->cfg.max_rows + 16 +
+                                                     m->lay.hist_slots * m->cfg.max_rows);
+            int32_t* hg = m->h_buf + m->cfg.max_seq;
+            KS_CUDA(cudaMemcpyAsync(hm, m->mask_dev, nsub, cudaMemcpyDeviceToHost, m->stream), "mask download");
+            KS_CUDA(cudaMemcpyAsync(hg, m->tpt_info, sizeof(int32_t) * 2, cudaMemcpyDeviceToHost, m->stream),
+                    "gamma download");
+            m->d2h += nsub + 2 * sizeof(int32_t);
+            KS_TRY(sync(m, "select"));
+            std::memcpy(mask.data(), hm, nsub);
+            gamma = hg[1];
+            st.resolves++;
+        }
         if (prm->policy == 1 && st.steps % prm->resolve_every == 0) {
             KS_TRY(ks_history_similarities(m, m->sims, nullptr));
             KS_TRY(launch(m, K_ACCEPT, [&] {
@@ -1038,7 +1245,7 @@ ks_status ks_generate_speculative(ks_model* m, const ks_spec_params* prm, int32_
             std::memcpy(mask.data(), hm, nsub);
             st.resolves++;
         }
-        int g = prm->gamma;
+        int g = gamma;
         if (m->p + g + 1 > m->cfg.max_seq) g = m->cfg.max_seq - m->p - 1;
         if (g < 1) {
             set_error("ks_generate_speculative: KV capacity exhausted");

@@ -71,6 +71,7 @@ cudaError_t launch_cosine(const void* X, const void* Y, int dtype, int64_t n_pai
 
 // ----------------------------------------------------------------- knapsack
 constexpr int kMaxItems = 256;
+constexpr int kMaxTpt = KS_TPT_MAX_CANDIDATES;
 constexpr int kKnapThreads = 512;
 
 struct KnapArgs {
@@ -89,12 +90,15 @@ struct KnapArgs {
     long long* best;          // scratch [2][cap + 1]
     uint8_t* take;            // scratch [n_items][cap + 1]
     int cap;                  // capacity of the scratch tables
+    int n_frontier;           // > 0: also backtrack the optima of budgets floor(sum w (j + 1) / n_frontier)
+    uint8_t* frontier;        // [n_frontier][n_items] masks of those budgets
 };
 
 __global__ void __launch_bounds__(kKnapThreads) knapsack_kernel(const KnapArgs a) {
     __shared__ int w[kMaxItems];
     __shared__ long long q[kMaxItems];
     __shared__ int B;
+    __shared__ long long SW;
     const int tid = threadIdx.x;
     const int N = a.n_items;
     if (tid == 0) {
@@ -117,6 +121,7 @@ __global__ void __launch_bounds__(kKnapThreads) knapsack_kernel(const KnapArgs a
             w[i] = (a.kind == 0) ? ((i % 2 == 0) ? wa : wm) : a.units[i];
             sum += w[i];
         }
+        SW = sum;
         long long b = a.budget;
         if (a.budget_frac >= 0.0) b = (long long)floor(__dmul_rn(a.budget_frac, (double)sum));
         if (b > a.cap) b = a.cap;
@@ -166,6 +171,19 @@ __global__ void __launch_bounds__(kKnapThreads) knapsack_kernel(const KnapArgs a
         }
         if (a.objective) *a.objective = (double)cur[B] / 1073741824.0;
     }
+    // The TPT stage's candidate set: the optimum of each frontier budget,
+    // backtracked from the same table (the DP up to capacity c does not
+    // depend on larger capacities).
+    for (int j = tid; j < a.n_frontier; j += blockDim.x) {
+        int c = (int)((SW * (long long)(j + 1)) / a.n_frontier);
+        if (c > B) c = B;
+        uint8_t* fm = a.frontier + (size_t)j * N;
+        for (int i = N - 1; i >= 0; --i) {
+            const uint8_t t = a.take[(size_t)i * (a.cap + 1) + c];
+            fm[i] = t;
+            if (t) c -= w[i];
+        }
+    }
     if (a.weights_out)
         for (int i = tid; i < N; i += blockDim.x) a.weights_out[i] = w[i];
 }
@@ -178,7 +196,8 @@ size_t select_scratch_bytes(int n_items, int cap) {
 
 cudaError_t launch_select(const ks_latency* lat, const float* sims, int64_t n, int n_items, int budget,
                           double budget_frac, uint8_t* mask, double* objective, int32_t* weights,
-                          int32_t* budget_out, void* scratch, int cap, cudaStream_t s) {
+                          int32_t* budget_out, void* scratch, int cap, cudaStream_t s, int n_frontier,
+                          uint8_t* frontier) {
     KnapArgs a{};
     a.kind = lat->kind;
     a.c1 = lat->c1;
@@ -198,7 +217,110 @@ cudaError_t launch_select(const ks_latency* lat, const float* sims, int64_t n, i
     a.cap = cap;
     a.best = reinterpret_cast<long long*>(scratch);
     a.take = reinterpret_cast<uint8_t*>(scratch) + sizeof(long long) * 2 * ((size_t)cap + 1);
+    a.n_frontier = n_frontier;
+    a.frontier = frontier;
     knapsack_kernel<<<1, kKnapThreads, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- TPT stage
+// Alg. 2 after the frontier: Eq. 4's acceptance of each candidate on the
+// history rows (its predicted tokens against the full layer set's), then the
+// grid search of Eq. 3 over candidates (in order) x gamma = 1..D, a pair
+// replacing the best only when its TPT is strictly larger.  Double
+// arithmetic with explicit round-to-nearest operations in a fixed order.
+struct TptArgs {
+    int kind;                 // 0 latency model, 1 explicit units
+    double c1, c2, c3;
+    long long n;
+    int units[kMaxItems];
+    int n_items, n_layers;
+    int K, r, D;
+    const uint8_t* frontier;  // [K][n_items]
+    const int32_t* tokens;    // [(K + 1) r]: candidate j's rows at j r, the full set's at K r
+    uint8_t* mask_out;        // [n_items] the chosen candidate
+    int32_t* info;            // [0] chosen candidate, [1] gamma
+    double* out;              // [0] TPT, [1 + j] alpha of candidate j
+};
+
+__global__ void __launch_bounds__(256) tpt_kernel(const TptArgs a) {
+    __shared__ double alpha[kMaxTpt];
+    __shared__ int sel;
+    const int tid = threadIdx.x;
+    for (int j = tid; j < a.K; j += blockDim.x) {
+        int cnt = 0;
+        for (int i = 0; i < a.r; ++i) cnt += a.tokens[(size_t)j * a.r + i] == a.tokens[(size_t)a.K * a.r + i];
+        alpha[j] = __ddiv_rn((double)cnt, (double)a.r);
+        a.out[1 + j] = alpha[j];
+    }
+    __syncthreads();
+    if (tid == 0) {
+        double ta = 0.0, tm = 0.0, tt = 0.0;
+        if (a.kind == 0) {
+            ta = __dadd_rn(__dmul_rn(a.c2, (double)a.n), a.c3);
+            tm = a.c1;
+            tt = __dmul_rn((double)a.n_layers, __dadd_rn(ta, tm));
+        } else {
+            for (int i = 0; i < a.n_items; ++i) tt = __dadd_rn(tt, (double)a.units[i]);
+        }
+        int bj = -1, bg = 0;
+        double bv = 0.0;
+        for (int j = 0; j < a.K; ++j) {
+            const uint8_t* m = a.frontier + (size_t)j * a.n_items;
+            double td = 0.0;
+            if (a.kind == 0) {
+                int na = 0, nm = 0;
+                for (int i = 0; i < a.n_items; ++i)
+                    if (m[i]) (i % 2 == 0 ? na : nm)++;
+                td = __dadd_rn(__dmul_rn((double)na, ta), __dmul_rn((double)nm, tm));
+            } else {
+                for (int i = 0; i < a.n_items; ++i)
+                    if (m[i]) td = __dadd_rn(td, (double)a.units[i]);
+            }
+            double e = 1.0, p = 1.0;
+            for (int g = 1; g <= a.D; ++g) {
+                p = __dmul_rn(p, alpha[j]);
+                e = __dadd_rn(e, p);   // Eq. 1 summed term by term
+                const double v = __ddiv_rn(e, __dadd_rn(__dmul_rn((double)g, td), tt));
+                if (v > bv) {
+                    bv = v;
+                    bj = j;
+                    bg = g;
+                }
+            }
+        }
+        a.info[0] = bj;
+        a.info[1] = bg;
+        a.out[0] = bv;
+        sel = bj;
+    }
+    __syncthreads();
+    for (int i = tid; i < a.n_items; i += blockDim.x) a.mask_out[i] = a.frontier[(size_t)sel * a.n_items + i];
+}
+
+cudaError_t launch_tpt(const ks_latency* lat, int64_t n, int n_items, int n_layers, int K, int r, int D,
+                       const uint8_t* frontier, const int32_t* tokens, uint8_t* mask_out, int32_t* info,
+                       double* out, cudaStream_t s) {
+    if (K < 1 || K > kMaxTpt || r < 1 || D < 1 || n_items > kMaxItems) return cudaErrorInvalidValue;
+    TptArgs a{};
+    a.kind = lat->kind;
+    a.c1 = lat->c1;
+    a.c2 = lat->c2;
+    a.c3 = lat->c3;
+    a.n = n;
+    if (lat->kind == 1)
+        for (int i = 0; i < n_items; ++i) a.units[i] = lat->units[i];
+    a.n_items = n_items;
+    a.n_layers = n_layers;
+    a.K = K;
+    a.r = r;
+    a.D = D;
+    a.frontier = frontier;
+    a.tokens = tokens;
+    a.mask_out = mask_out;
+    a.info = info;
+    a.out = out;
+    tpt_kernel<<<1, 256, 0, s>>>(a);
     return cudaGetLastError();
 }
 

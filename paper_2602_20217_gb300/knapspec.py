@@ -47,7 +47,7 @@ class KsLatency(C.Structure):
 class KsSpecParams(C.Structure):
     _fields_ = [("gamma", C.c_int32), ("policy", C.c_int32), ("mask", C.POINTER(C.c_uint8)),
                 ("latency", KsLatency), ("budget_frac", C.c_double), ("resolve_every", C.c_int32),
-                ("max_steps", C.c_int32)]
+                ("max_steps", C.c_int32), ("tpt_candidates", C.c_int32), ("tpt_max_gamma", C.c_int32)]
 
 
 class KsSpecStats(C.Structure):
@@ -88,6 +88,8 @@ _SIGS = {
     "ks_debug_read": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32, C.c_int32, C.c_int32, C.c_void_p, C.c_size_t]),
     "ks_kernel_timing": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32]),
     "ks_kernel_time": (C.c_int, [C.c_void_p, C.c_int32, C.POINTER(C.c_int64), C.POINTER(C.c_double)]),
+    "ks_select_tpt": (C.c_int, [C.c_void_p, C.POINTER(KsLatency), C.c_int32, C.c_int32, C.c_void_p,
+                                C.POINTER(C.c_int32), C.POINTER(C.c_double), C.c_void_p, C.c_void_p]),
     "ks_kernel_bytes": (C.c_int, [C.c_void_p, C.c_int32, C.POINTER(C.c_double)]),
     "ks_launch_count": (C.c_int64, [C.c_void_p]),
     "ks_transfer_bytes": (C.c_int, [C.c_void_p, C.POINTER(C.c_int64), C.POINTER(C.c_int64)]),
@@ -299,6 +301,18 @@ def ks_kernel_bytes(h: int, klass: int) -> float:
     b = C.c_double()
     check(load().ks_kernel_bytes(h, klass, C.byref(b)), "ks_kernel_bytes")
     return b.value
+
+
+def ks_select_tpt(h: int, lat: "KsLatency", n_sublayers: int, n_candidates: int, max_gamma: int):
+    """TPT stage on the model's history: (mask, gamma, tpt, alphas, candidates)."""
+    mask = np.zeros(n_sublayers, np.uint8)
+    cand = np.zeros((n_candidates, n_sublayers), np.uint8)
+    alphas = np.zeros(n_candidates, np.float64)
+    g = C.c_int32()
+    t = C.c_double()
+    check(load().ks_select_tpt(h, C.byref(lat), n_candidates, max_gamma, mask.ctypes.data, C.byref(g),
+                               C.byref(t), alphas.ctypes.data, cand.ctypes.data), "ks_select_tpt")
+    return mask, g.value, t.value, alphas, cand
 
 
 def ks_launch_count(h: int) -> int:

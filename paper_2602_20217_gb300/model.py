@@ -48,8 +48,10 @@ class Model:
         return ks.ks_model_position(self.h)
 
     def generate(self, n_tokens: int, gamma: int, mask=None, latency=None, budget_frac: float = 0.5,
-                 resolve_every: int = 64, max_steps: int = 0):
-        """Speculative decoding: a fixed mask (policy 0) or the knapsack policy."""
+                 resolve_every: int = 64, max_steps: int = 0, tpt=None):
+        """Speculative decoding: a fixed mask (policy 0), the knapsack policy
+        (policy 1, latency given) or the TPT stage (policy 2, latency and
+        tpt = (n_candidates, max_gamma) given)."""
         n = self.shape.n_sublayers
         keep = []
         if latency is None:
@@ -60,8 +62,17 @@ class Model:
         else:
             lat, u = latency
             keep.append(u)
-            p = ks.KsSpecParams(gamma, 1, None, lat, float(budget_frac), int(resolve_every), max_steps)
+            if tpt is None:
+                p = ks.KsSpecParams(gamma, 1, None, lat, float(budget_frac), int(resolve_every), max_steps)
+            else:
+                p = ks.KsSpecParams(gamma, 2, None, lat, 0.0, int(resolve_every), max_steps,
+                                    int(tpt[0]), int(tpt[1]))
         return ks.ks_generate_speculative(self.h, p, n_tokens)
+
+    def select_tpt(self, latency, n_candidates: int, max_gamma: int):
+        """The TPT stage on the current history: (mask, gamma, tpt, alphas, candidates)."""
+        lat, _u = latency
+        return ks.ks_select_tpt(self.h, lat, self.shape.n_sublayers, n_candidates, max_gamma)
 
     def history_similarities(self):
         import torch

@@ -93,6 +93,10 @@ def test_error_paths_touch_no_device(lib):
     assert lib.ks_decode_greedy(None, 4, out.ctypes.data) == ks.KS_ERR_INVALID_ARG
     assert lib.ks_model_destroy(None) == ks.KS_ERR_INVALID_ARG
     assert lib.ks_launch_count(None) == -1
+    lat, _ = ks.latency(0, 1.0, 0.0, 1.0)
+    g, t = C.c_int32(), C.c_double()
+    assert lib.ks_select_tpt(None, C.byref(lat), 4, 4, out.ctypes.data, C.byref(g), C.byref(t), None,
+                             None) == ks.KS_ERR_INVALID_ARG
 
 
 def test_select_mask_argument_checks(lib):
