@@ -211,7 +211,8 @@ def gpu_arm(args):
     sh = wl.shape
     gamma = args.gamma or wl.gammas[len(wl.gammas) // 2]
     prompt = synth.prompt_tokens(sh, wl.prompt_len, seed=wl.prompt_seed)
-    max_seq = wl.prompt_len + (max(args.steps, args.warmup) + 2) * (gamma + 1) + args.e2e_tokens + 64
+    g_max = max(gamma, int(args.tpt_max_gamma)) if args.policy == "tpt" or args.sweep else gamma
+    max_seq = wl.prompt_len + (max(args.steps, args.warmup) + 2) * (g_max + 1) + args.e2e_tokens + 64
     t0 = time.time()
     model = Model(sh, max_seq=max_seq, seed=wl.weight_seed)
     torch.cuda.synchronize()
@@ -246,7 +247,12 @@ def gpu_arm(args):
     c2 = per("attn") / wl.prompt_len
     lat, _keep = ks.latency(0, c1, c2, c3)
 
+    tpt_d = int(args.tpt_max_gamma)   # D of Alg. 2: the longest draft the grid search may pick
+
     def params(max_steps):
+        if args.policy == "tpt":
+            return ks.KsSpecParams(gamma, 2, None, lat, 0.0, int(args.tpt_every), int(max_steps),
+                                   int(args.tpt_candidates), tpt_d)
         return ks.KsSpecParams(gamma, 1, None, lat, float(args.budget_frac), int(args.resolve_every),
                                int(max_steps))
 
@@ -322,6 +328,16 @@ def gpu_arm(args):
                               "alpha": float(sst.accepted) / max(1, sst.drafted),
                               "tokens_per_step": n_tok / max(1, sst.steps),
                               "skipped_attn_mlp": [int(sst.attn_skipped), int(sst.mlp_skipped)]})
+        # the TPT stage (Alg. 2) picks the layer set and gamma itself
+        p = ks.KsSpecParams(gamma, 2, None, lat, 0.0, int(args.tpt_every), 0, int(args.tpt_candidates), tpt_d)
+        (o, sst, _a), t = timed(lambda: ks.ks_generate_speculative(h, p, args.e2e_tokens))
+        n_tok = int(sst.steps + sst.accepted)
+        sweep.append({"policy": f"tpt every {args.tpt_every} steps, K {args.tpt_candidates}, D {tpt_d}",
+                      "tokens_per_s": n_tok / t, "vs_greedy": (n_tok / t) / ((args.e2e_tokens - 1) / t_ar),
+                      "alpha": float(sst.accepted) / max(1, sst.drafted),
+                      "mean_gamma": float(sst.drafted) / max(1, sst.steps),
+                      "tokens_per_step": n_tok / max(1, sst.steps),
+                      "skipped_attn_mlp": [int(sst.attn_skipped), int(sst.mlp_skipped)]})
 
     ms_max, tok_all = reduce_over_ranks(ms, tokens, dist, "cuda")
 
@@ -337,11 +353,14 @@ def gpu_arm(args):
             "data": "synthetic (seeded random-init weights, uniform random prompt ids)",
             "config": {"workload": wl.name, "model": sh.name, "prompt": wl.prompt_len, "gamma": gamma,
                        "policy": (f"knapsack re-solved every {args.resolve_every} step(s), "
-                                  f"budget {args.budget_frac} of sum w"),
+                                  f"budget {args.budget_frac} of sum w") if args.policy == "knapsack" else
+                                 (f"TPT stage every {args.tpt_every} step(s), K {args.tpt_candidates}, "
+                                  f"D {tpt_d}"),
                        "l2": "inputs larger than L2 (each step streams the weights, 16+ GB)",
                        "parallelism": f"replicas x{world}"},
             "tokens": tokens, "mean_tokens_per_step": tokens / max(1, st.steps),
             "alpha": float(st.accepted) / max(1, st.drafted),
+            "mean_gamma": float(st.drafted) / max(1, st.steps),
             "mask_skipped": {"attn": int(st.attn_skipped), "mlp": int(st.mlp_skipped)},
             "ar_tokens_per_s": (args.e2e_tokens - 1) / ar_s,
             "spec_vs_ar_e2e": (e2e_tok / e2e_s) / ((args.e2e_tokens - 1) / ar_s),
@@ -386,6 +405,12 @@ def main():
     ap.add_argument("--resolve-every", dest="resolve_every", type=int, default=1)
     ap.add_argument("--e2e-tokens", dest="e2e_tokens", type=int, default=256)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--policy", default="knapsack", choices=["knapsack", "tpt"],
+                    help="mask policy of the timed steps: knapsack at --budget-frac, or the TPT stage")
+    ap.add_argument("--tpt-every", dest="tpt_every", type=int, default=8)
+    ap.add_argument("--tpt-candidates", dest="tpt_candidates", type=int, default=8)
+    ap.add_argument("--tpt-max-gamma", dest="tpt_max_gamma", type=int, default=7,
+                    help="D of Alg. 2 (1..15); the default keeps verify passes at 8 rows or fewer")
     ap.add_argument("--sweep", action="store_true",
                     help="also time jobs over a grid of knapsack budgets and draft lengths")
     ap.add_argument("--sweep-budgets", dest="sweep_budgets", default="0.4,0.5,0.6,0.7,0.8")

@@ -62,6 +62,13 @@ constexpr size_t kRingBudget1 = 196u * 1024u;        // one CTA per SM
 constexpr size_t kRingBudget2 = 104u * 1024u;        // two CTAs per SM
 constexpr int kMaxRows = 16;
 
+// Status word codes (the first one recorded stays): a bounded wait ran out,
+// or a self-check found a stage or item record out of range (the access it
+// guards is skipped).
+constexpr int kErrWait = 1;
+constexpr int kErrCheckW = 2, kErrCheckA = 3, kErrCheckC = 4, kErrCheckE = 5;
+KS_DEV void set_err(int* e, int code) { atomicCAS(e, 0, code); }
+
 struct Phase {
     int kind, layer, N, K, n_items, tpi;
 };
@@ -289,6 +296,11 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
             int t = 0;
             auto issue = [&](int k, const Phase& P, int it, int kt, bool last_item) -> bool {
                 const int slot = t % S;
+                // self-check: every box coordinate below follows from these ranges
+                if (k < 0 || k >= a.n_phases || it < 0 || it >= P.n_items || kt < 0 || kt >= P.tpi) {
+                    set_err(a.err, kErrCheckW);
+                    return false;
+                }
                 if (t >= S && !mbar_wait(&empty[slot], (uint32_t)(((t / S) - 1) & 1), kWaitLimitNs)) return false;
                 slot_k[slot] = k;
                 slot_it[slot] = it;
@@ -348,7 +360,7 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
                     mbar_arrive(&pub[slot]);
                 }
             }
-            if (!ok) atomicExch(a.err, 1);
+            if (!ok) set_err(a.err, kErrWait);
             // (a dependent launch starts only after this grid's predecessor
             // completed, so the alternating counter sets never overlap)
             grid_dependency_wait();
@@ -375,7 +387,17 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
                 break;
             }
             const int kt = slot_kt[slot];
+            if (k >= a.n_phases || kt < 0) {   // self-check of the stage record
+                if (lane == 0) set_err(a.err, kErrCheckA);
+                ok = false;
+                break;
+            }
             const Phase P = decode(a, k);
+            if (kt >= P.tpi) {
+                if (lane == 0) set_err(a.err, kErrCheckA);
+                ok = false;
+                break;
+            }
             if (k != cur) {
                 cur = k;
                 ready = 0;      // blocks of phase k - 1 known to be complete
@@ -426,7 +448,7 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
             }
             __syncwarp();
         }
-        if (!ok && lane == 0) atomicExch(a.err, 1);
+        if (!ok && lane == 0) set_err(a.err, kErrWait);
     } else if (warp < 4) {
         // ------------------------------------------------------ consumers
         float acc[kChains][NT][4], accu[kChains][NT][4];
@@ -452,7 +474,17 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
                 if (lane == 0) mbar_arrive(&red_full[b]);
                 break;
             }
+            if (k >= a.n_phases || kt < 0 || it < 0) {   // self-check (the same record in every warp)
+                if (lane == 0) set_err(a.err, kErrCheckC);
+                failed = true;
+                break;
+            }
             const Phase P = decode(a, k);
+            if (kt >= P.tpi || it >= P.n_items) {
+                if (lane == 0) set_err(a.err, kErrCheckC);
+                failed = true;
+                break;
+            }
             if (kt == 0) {
 #pragma unroll
                 for (int c = 0; c < kChains; ++c)
@@ -500,7 +532,7 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
             if (lane == 0) mbar_arrive(&red_full[b]);
             ++n_items;
         }
-        if (failed && lane == 0) atomicExch(a.err, 1);
+        if (failed && lane == 0) set_err(a.err, kErrWait);
     } else if (warp == kWarpE) {
         // --------------------------------------------------- epilogue warp
         grid_dependency_wait();   // epilogues write buffers the previous kernel uses
@@ -526,6 +558,11 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
             if (k < 0) break;
             const int it = red_it[b];
             const bool last_item = red_last[b] != 0;
+            if (k >= a.n_phases || it < 0 || it >= decode(a, k).n_items) {   // self-check
+                set_err(a.err, kErrCheckE);
+                ok = false;
+                break;
+            }
             const Phase P = decode(a, k);
             // the four warps' K quarters, added in warp order
 #pragma unroll
@@ -591,7 +628,7 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
                 }
             }
         }
-        if (!ok && lane == 0) atomicExch(a.err, 1);
+        if (!ok && lane == 0) set_err(a.err, kErrWait);
     }
 
     // the last CTA to leave resets the queues and counters for the next launch

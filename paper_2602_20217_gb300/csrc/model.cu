@@ -553,9 +553,13 @@ static ks_status sync(ks_model* m, const char* what) {
     if (e != cudaSuccess) return cuda_fail(e, what);
     e = cudaStreamSynchronize(m->stream);
     if (e != cudaSuccess) return cuda_fail(e, what);
-    if (*hs != 0) {
+    if (*hs == 1) {
         set_error("%s: a kernel gave up waiting for an asynchronous copy", what);
         return KS_ERR_TIMEOUT;
+    }
+    if (*hs != 0) {
+        set_error("%s: a kernel's self-check failed (status word %d)", what, *hs);
+        return KS_ERR_STATE;
     }
     return KS_OK;
 }
