@@ -103,7 +103,15 @@ def run_oracle_arm(args, workload):
     return float(np.mean(samples))
 
 
-def cpu_baseline(workload: str, steps: int = 1, warmup: int = 0) -> dict:
+_T0 = time.time()
+
+
+def progress(msg: str):
+    """One timestamped line on stderr per bench stage (the JSON line stays alone on stdout)."""
+    print(f"[bench {time.time() - _T0:7.1f}s] {msg}", file=sys.stderr, flush=True)
+
+
+def cpu_baseline(workload: str, steps: int = 1, warmup: int = 0, timeout: float = 300.0) -> dict:
     cores = os.cpu_count() or 1
     env = dict(os.environ)
     for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
@@ -111,7 +119,7 @@ def cpu_baseline(workload: str, steps: int = 1, warmup: int = 0) -> dict:
     code = ("import sys, json; sys.path.insert(0, %r); import bench; "
             "print(json.dumps(bench.run_oracle_arm(type('A', (), {'steps': %d, 'warmup': %d})(), %r)))"
             % (ROOT, steps, warmup, workload))
-    out = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True, timeout=900)
+    out = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True, timeout=timeout)
     if out.returncode != 0:
         raise RuntimeError("oracle baseline failed: " + out.stderr[-2000:])
     t_token = float(out.stdout.strip().splitlines()[-1])
@@ -233,7 +241,9 @@ def gpu_arm(args):
     # c1 = MLP sublayer (gate/up + down), c3 = the Attn sublayer's
     # context-independent kernels (QKV, merge, O-proj), c2 = attention-kernel
     # time / context length.
+    progress("model created; prefill")
     t_prefill = prefill()
+    progress("prefill done; latency model")
     split = [k for name, k in ks.KLASS.items() if name != "chain"]   # one projection per launch
     for k in split:
         ks.ks_kernel_timing(h, k, True)
@@ -257,6 +267,7 @@ def gpu_arm(args):
                                int(max_steps))
 
     # warm-up
+    progress("warm-up")
     rewind()
     ks.ks_generate_speculative(h, params(args.warmup), 1 << 30)
     # timed region: exactly K speculation steps, device time on the model's stream
@@ -292,6 +303,7 @@ def gpu_arm(args):
     rewind()
     h2d0, d2h0 = ks.ks_transfer_bytes(h)
     t0 = time.perf_counter()
+    progress("timed region done; end-to-end job")
     out, est, eacc = ks.ks_generate_speculative(h, params(0), args.e2e_tokens)
     e2e_s = time.perf_counter() - t0
     h2d1, d2h1 = ks.ks_transfer_bytes(h)
@@ -299,7 +311,9 @@ def gpu_arm(args):
     # the same library's plain greedy decode of the same job
     rewind()
     t0 = time.perf_counter()
+    progress("greedy job")
     ar = ks.ks_decode_greedy(h, args.e2e_tokens)
+    progress("greedy job done")
     ar_s = time.perf_counter() - t0
     lossless = bool(np.array_equal(out, ar))
 
@@ -384,6 +398,7 @@ def gpu_arm(args):
             line["sweep_device_time"] = sweep
         if not args.no_cpu_baseline and world == 1:
             try:
+                progress("oracle baseline")
                 line["cpu_baseline"] = cpu_baseline(wl.name)
             except Exception as e:  # reported, never hidden
                 line["cpu_baseline"] = {"error": str(e)[:300]}
