@@ -24,6 +24,12 @@ Readings where the paper is silent (each listed in the design notes):
 * Greedy argmax breaks ties towards the lowest token id.
 * History: the committed rows of each verify step form one entry; the prompt's
   last ``hist_init_rows`` rows form the first entry; the last m entries are kept.
+* Dynamic drafting exit (Sec. 3.5, "Dynamic Drafting Exit"): the confidence of
+  a draft token is the softmax probability of its argmax over the draft's
+  logits; drafting stops after the first token whose confidence is below
+  tau_conf, and that token stays the step's last draft (its verification costs
+  nothing extra).  The confidence is exp(l_max) / sum_i exp(l_i), computed as
+  1 / sum_i exp(l_i - l_max).
 """
 from __future__ import annotations
 
@@ -143,6 +149,13 @@ def greedy(logits: np.ndarray) -> np.ndarray:
     return np.argmax(logits, axis=-1).astype(np.int64)
 
 
+def top1_prob(logits_row: np.ndarray) -> float:
+    """Softmax probability of the argmax token of one row of logits (the
+    draft confidence of Sec. 3.5): 1 / sum_i exp(l_i - max_j l_j)."""
+    l = np.asarray(logits_row, dtype=np.float64)
+    return float(1.0 / np.sum(np.exp(l - np.max(l))))
+
+
 def as_f64(weights: dict) -> dict:
     """Widen a weight dict (fp32 / bf16 values held as fp32) to fp64."""
     out = {k: np.asarray(v, np.float64) for k, v in weights.items() if k != "layers"}
@@ -220,14 +233,22 @@ class Session:
         self.pending = int(greedy(logits)[0])
         return self.pending
 
-    def draft(self, mask, gamma: int) -> list:
-        """gamma greedy tokens from f^(S) starting at the pending token (Sec. 2.2)."""
+    def draft(self, mask, gamma: int, tau_conf: float | None = None) -> list:
+        """Up to gamma greedy tokens from f^(S) starting at the pending token
+        (Sec. 2.2).  With tau_conf, drafting stops after the first token whose
+        top-1 probability is below tau_conf (Sec. 3.5, dynamic drafting exit).
+        The confidence of every drafted token is left in ``last_confidence``."""
         tok = self.pending
         out = []
+        self.last_confidence = []
         for t in range(gamma):
             logits, _ = self.forward([tok], self.p + t, mask=mask)
             tok = int(greedy(logits)[0])
             out.append(tok)
+            c = top1_prob(logits[0])
+            self.last_confidence.append(c)
+            if tau_conf is not None and c < tau_conf:
+                break
         return out
 
     def verify(self, drafts) -> tuple:
@@ -263,12 +284,13 @@ def greedy_generate(cfg, weights, prompt, n_new: int, n_max: int | None = None) 
 
 
 def spec_generate(cfg, weights, prompt, n_new: int, gamma: int, choose_mask,
-                  n_max: int | None = None, resolve_every: int = 1):
+                  n_max: int | None = None, resolve_every: int = 1, tau_conf: float | None = None):
     """Greedy self-speculative decoding.
 
     ``choose_mask(session)`` returns the draft mask; it is called before the
-    first step and again every ``resolve_every`` verify steps.  Returns
-    (tokens, per-step accepted counts, masks used)."""
+    first step and again every ``resolve_every`` verify steps.  ``tau_conf``
+    enables the dynamic drafting exit (Sec. 3.5).  Returns (tokens, per-step
+    accepted counts, masks used)."""
     n_max = n_max or (len(prompt) + n_new + gamma + 2)
     s = Session(cfg, weights, n_max)
     out = [s.prefill(prompt)]
@@ -279,7 +301,7 @@ def spec_generate(cfg, weights, prompt, n_new: int, gamma: int, choose_mask,
         if step % resolve_every == 0:
             mask = choose_mask(s)
         g = min(gamma, n_max - s.p - 1)
-        drafts = s.draft(mask, g)
+        drafts = s.draft(mask, g, tau_conf)
         a, new = s.verify(drafts)
         out.extend(new)
         accepted.append(a)

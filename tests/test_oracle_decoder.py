@@ -281,3 +281,57 @@ def test_history_ring_holds_committed_rows():
     # X^(0) of the newest entry = embeddings of that step's committed tokens
     committed = [before] + drafts[:a]
     assert np.array_equal(s.history()[0, -(a + 1):], w["embed"][committed])
+
+
+def test_top1_prob_closed_forms():
+    # Sec. 3.5 confidence = softmax probability of the argmax token
+    assert abs(D.top1_prob(np.full(1000, 3.7)) - 1e-3) < 1e-15          # uniform: 1 / V
+    assert abs(D.top1_prob(np.array([np.log(3.0), 0.0])) - 0.75) < 1e-15  # 3 / (3 + 1)
+    assert D.top1_prob(np.array([5.0, 5.0, -800.0, -800.0])) == 0.5      # two tied maxima
+    assert D.top1_prob(np.array([0.0, 0.0, 0.0, 800.0])) == 1.0           # one dominant logit
+    l = np.random.default_rng(0).normal(size=257)
+    p = D.top1_prob(l)
+    assert abs(D.top1_prob(l + 1234.5) - p) < 1e-12                      # shift invariance
+    l2 = l.copy()
+    l2[np.argmax(l)] += 0.5
+    assert D.top1_prob(l2) > p                                            # a larger max is more confident
+    # brute force in exact rationals: logits log(k) give probabilities k / sum(k)
+    ks = np.arange(1, 9, dtype=np.float64)
+    assert abs(D.top1_prob(np.log(ks)) - 8.0 / 36.0) < 1e-15
+
+
+def test_dynamic_exit_stops_after_first_unconfident_token():
+    cfg = tiny_cfg(L=3)
+    w = rand_weights(cfg, seed=21, std=0.6)
+    prompt = np.random.default_rng(22).integers(0, cfg.vocab, 14)
+    mask = np.array([1, 0, 1, 1, 0, 1], np.uint8)
+    s = D.Session(cfg, w, 64)
+    s.prefill(prompt)
+    full = s.draft(mask, 6)                       # no exit: gamma tokens
+    conf = list(s.last_confidence)
+    assert len(full) == 6 and len(conf) == 6
+    # the recorded confidence is top1_prob of the draft's own logits
+    s2 = D.Session(cfg, w, 64)
+    s2.prefill(prompt)
+    logits, _ = s2.forward([s2.pending], s2.p, mask=mask)
+    assert abs(conf[0] - D.top1_prob(logits[0])) < 1e-15
+    for tau in (0.0, 1.01, *sorted(conf)):
+        s3 = D.Session(cfg, w, 64)
+        s3.prefill(prompt)
+        got = s3.draft(mask, 6, tau)
+        below = [i for i, c in enumerate(conf) if c < tau]
+        n = below[0] + 1 if below else 6          # the unconfident token is kept, then drafting stops
+        assert got == full[:n], (tau, got, full)
+
+
+@pytest.mark.parametrize("tau", [0.0, 0.2, 0.5, 1.01])
+def test_lossless_with_dynamic_exit(tau):
+    cfg = tiny_cfg(qk_norm=True, L=3)
+    w = rand_weights(cfg, seed=23, std=0.6)
+    prompt = np.random.default_rng(24).integers(0, cfg.vocab, 16)
+    mask = np.array([0, 1, 1, 1, 0, 1], np.uint8)
+    ar = D.greedy_generate(cfg, w, prompt, 24)
+    toks, acc, _ = D.spec_generate(cfg, w, prompt, 24, 5, lambda s: mask, tau_conf=tau)
+    assert toks == ar
+    if tau > 1.0:
+        assert all(a <= 1 for a in acc)           # one draft per step
