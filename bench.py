@@ -262,9 +262,9 @@ def gpu_arm(args):
     def params(max_steps):
         if args.policy == "tpt":
             return ks.KsSpecParams(gamma, 2, None, lat, 0.0, int(args.tpt_every), int(max_steps),
-                                   int(args.tpt_candidates), tpt_d)
+                                   int(args.tpt_candidates), tpt_d, float(args.tau_conf))
         return ks.KsSpecParams(gamma, 1, None, lat, float(args.budget_frac), int(args.resolve_every),
-                               int(max_steps))
+                               int(max_steps), 0, 0, float(args.tau_conf))
 
     # warm-up
     progress("warm-up")
@@ -352,6 +352,15 @@ def gpu_arm(args):
                       "mean_gamma": float(sst.drafted) / max(1, sst.steps),
                       "tokens_per_step": n_tok / max(1, sst.steps),
                       "skipped_attn_mlp": [int(sst.attn_skipped), int(sst.mlp_skipped)]})
+        # the dynamic drafting exit of Sec. 3.5 (tau_conf 0.7) on the default knapsack policy
+        p = ks.KsSpecParams(gamma, 1, None, lat, float(args.budget_frac), int(args.resolve_every), 0, 0, 0, 0.7)
+        (o, sst, _a), t = timed(lambda: ks.ks_generate_speculative(h, p, args.e2e_tokens))
+        n_tok = int(sst.steps + sst.accepted)
+        sweep.append({"policy": f"knapsack, gamma {gamma} max, budget {args.budget_frac}, dynamic exit tau_conf 0.7",
+                      "tokens_per_s": n_tok / t, "vs_greedy": (n_tok / t) / ((args.e2e_tokens - 1) / t_ar),
+                      "alpha": float(sst.accepted) / max(1, sst.drafted),
+                      "drafts_per_step": float(sst.drafted) / max(1, sst.steps),
+                      "tokens_per_step": n_tok / max(1, sst.steps)})
 
     ms_max, tok_all = reduce_over_ranks(ms, tokens, dist, "cuda")
 
@@ -366,10 +375,11 @@ def gpu_arm(args):
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": sh.dtype,
             "data": "synthetic (seeded random-init weights, uniform random prompt ids)",
             "config": {"workload": wl.name, "model": sh.name, "prompt": wl.prompt_len, "gamma": gamma,
-                       "policy": (f"knapsack re-solved every {args.resolve_every} step(s), "
+                       "policy": ((f"knapsack re-solved every {args.resolve_every} step(s), "
                                   f"budget {args.budget_frac} of sum w") if args.policy == "knapsack" else
                                  (f"TPT stage every {args.tpt_every} step(s), K {args.tpt_candidates}, "
-                                  f"D {tpt_d}"),
+                                  f"D {tpt_d}"))
+                                 + (f", dynamic exit tau_conf {args.tau_conf}" if args.tau_conf > 0 else ""),
                        "l2": "inputs larger than L2 (each step streams the weights, 16+ GB)",
                        "parallelism": f"replicas x{world}"},
             "tokens": tokens, "mean_tokens_per_step": tokens / max(1, st.steps),
@@ -424,6 +434,8 @@ def main():
                     help="mask policy of the timed steps: knapsack at --budget-frac, or the TPT stage")
     ap.add_argument("--tpt-every", dest="tpt_every", type=int, default=8)
     ap.add_argument("--tpt-candidates", dest="tpt_candidates", type=int, default=8)
+    ap.add_argument("--tau-conf", dest="tau_conf", type=float, default=0.0,
+                    help="dynamic drafting exit threshold (Sec. 3.5); 0 drafts gamma tokens every step")
     ap.add_argument("--tpt-max-gamma", dest="tpt_max_gamma", type=int, default=7,
                     help="D of Alg. 2 (1..15); the default keeps verify passes at 8 rows or fewer")
     ap.add_argument("--sweep", action="store_true",

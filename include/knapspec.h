@@ -152,6 +152,22 @@ ks_status ks_rewind(ks_model* m, int32_t* next_token);
  * is not NULL the call also waits for them and copies them out. */
 ks_status ks_draft(ks_model* m, const uint8_t* mask, int32_t gamma, int32_t* draft_tokens);
 
+/* a1 with the dynamic drafting exit of Sec. 3.5 ("Dynamic Drafting Exit"):
+ * like ks_draft with gamma as the maximum draft length, but after each draft
+ * token the device computes its confidence, the softmax probability of the
+ * token over the draft's logits, 1 / sum_i exp(l_i - l_max), and once a token's
+ * confidence is below tau_conf the step's remaining draft passes do nothing
+ * (that token stays the step's last draft).  tau_conf: finite, >= 0 (0 never
+ * stops; above 1 always stops after one token).  Everything stays on the
+ * device with no host synchronisation unless an output is requested; the
+ * following ks_verify (draft_tokens NULL, same gamma) still scores gamma + 1
+ * rows but compares only the drafts produced.
+ * Outputs (host, each optional; any of them makes the call wait): *n_drafted
+ * (1 .. gamma), confidence[0 .. n_drafted) (float; room for gamma), and
+ * draft_tokens[0 .. n_drafted) (room for gamma). */
+ks_status ks_draft_dynamic(ks_model* m, const uint8_t* mask, int32_t gamma, float tau_conf, int32_t* n_drafted,
+                           float* confidence, int32_t* draft_tokens);
+
 /* a2 + a3 (Sec. 2.1): score [pending, drafts...] (gamma + 1 rows at positions
  * p..p+gamma) with the full target in one pass, take the greedy argmax of
  * each row, accept the longest prefix of drafts equal to the target's
@@ -276,6 +292,8 @@ typedef struct {
     int32_t max_steps;       /* stop after this many verify steps (0: no limit)             */
     int32_t tpt_candidates;  /* policy 2: n_candidates of ks_select_tpt                     */
     int32_t tpt_max_gamma;   /* policy 2: max_gamma of ks_select_tpt                        */
+    double tau_conf;         /* > 0: dynamic drafting exit (ks_draft_dynamic) with this
+                                tau_conf; 0: every step drafts gamma tokens               */
 } ks_spec_params;
 
 typedef struct {

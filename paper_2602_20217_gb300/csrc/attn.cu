@@ -199,6 +199,7 @@ KS_DEV int my_chunk(const AttnArgs& a) {
 //   (K / V rows unpadded and chunk-swizzled, see kv_off).
 template <int HD>
 __global__ void __launch_bounds__(128) attn_bf16_kernel(const AttnArgs a) {
+    if (a.stop && *a.stop) return;   // a draft pass after the dynamic exit
     constexpr int NPL = HD / 32;
     constexpr int P = HD + 8;
     constexpr int NDT = HD / 8;  // dim tiles of 8
@@ -489,6 +490,7 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const AttnArgs a) {
 // fp32 models.
 template <int HD>
 __global__ void __launch_bounds__(128) attn_f32_kernel(const AttnArgs a) {
+    if (a.stop && *a.stop) return;   // a draft pass after the dynamic exit
     constexpr int NPL = HD / 32;
     constexpr int C = 2048;  // largest chunk of the schedule
     extern __shared__ float fsm[];
@@ -563,6 +565,7 @@ __global__ void __launch_bounds__(128) attn_f32_kernel(const AttnArgs a) {
 // same bits in a 1-row pass and in a gamma+1-row pass.
 template <typename WT, int HD>
 __global__ void __launch_bounds__(128) attn_merge_kernel(const AttnArgs a) {
+    if (a.stop && *a.stop) return;   // a draft pass after the dynamic exit
     extern __shared__ float wsh[];  // [nch] chunk weights
     __shared__ float red[kAttnWarps + 1];
     __shared__ float osh[kAttnWarps][HD];

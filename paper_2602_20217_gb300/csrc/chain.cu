@@ -252,6 +252,9 @@ KS_DEV void epilogue(const ChainArgs& a, const Phase& P, int k, int it, float (&
 
 template <int NT, int CTAS_PER_SM>
 __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __grid_constant__ ChainArgs a) {
+    // A draft pass after the dynamic exit: nothing to do.  The flag only
+    // changes between passes, so every CTA of the launch sees the same value.
+    if (a.stop && *a.stop) return;
     extern __shared__ unsigned char smem_raw[];
     // 1024-byte aligned: the 128-byte swizzle pattern repeats every 1024 bytes
     __nv_bfloat16* ring = reinterpret_cast<__nv_bfloat16*>(

@@ -279,6 +279,7 @@ KS_DEV void final_argmax(const GemvArgs& a, int groups) {
 // One CTA per (64-feature group, K slice); used for fp32 models only.
 template <int NT, int EPI>
 __global__ void __launch_bounds__(128) gemv_f32_kernel(const GemvArgs a) {
+    if (a.stop && *a.stop) return;   // a draft pass after the dynamic exit
     constexpr bool PAIR = (EPI == EPI_SWIGLU);
     extern __shared__ __align__(16) unsigned char smem[];
     __shared__ float red[kGemvWarps * kMaxRows + kMaxRows];

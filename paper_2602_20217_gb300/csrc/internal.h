@@ -34,6 +34,7 @@ struct GemvArgs {
     __nv_bfloat16* xg_out;  // EPI_RESID (bf16): new residual times next_gain, the next GEMV's input
     const void* next_gain;  // gain of the next RMSNorm (model dtype)
     int* err;               // device status word: set to 1 when a bounded wait gives up
+    const int* stop;        // draft passes: the pass is skipped when *stop != 0 (null: always run)
     float* out; int out_ld;                    // EPI_STORE (fp32)
     float* resid; int resid_ld;                // EPI_RESID: resid[r][n] += y
     float* capture; long long capture_ld;      // EPI_RESID: optional copy of the new residual
@@ -94,6 +95,7 @@ struct ChainArgs {
     long long capture_plane;
     int* counters;              // chain_counter_ints() zeros; the launch leaves them zero
     int* err;                   // device status word
+    const int* stop;            // draft passes: the launch does nothing when *stop != 0 (null: always)
     uint16_t code[kChainMaxPhases];
     const __nv_bfloat16* gain[kChainMaxPhases];  // O / down phases: gain of the next RMSNorm
 };
@@ -119,6 +121,7 @@ struct AttnArgs {
     int n_chunks_max;
     void* out;              // [R][hq hd] model dtype: merged attention output
     int out_ld;
+    const int* stop;        // draft passes: skipped when *stop != 0 (null: always run)
 };
 
 cudaError_t launch_attention(int dtype, const AttnArgs& a, cudaStream_t s);

@@ -43,7 +43,8 @@ enum { K_QKV = 0, K_ATTN, K_MERGE, K_OPROJ, K_GATEUP, K_DOWN, K_LMHEAD, K_EMBED,
 template <typename WT>
 __global__ void __launch_bounds__(256) embed_kernel(const WT* embed, const int32_t* tok, int d, int vocab, float* x,
                                                     float* capture, float* ss, __nv_bfloat16* xg,
-                                                    const WT* next_gain) {
+                                                    const WT* next_gain, const int* stop) {
+    if (stop && *stop) return;   // a draft pass after the dynamic exit
     const int r = blockIdx.x;
     const int k = blockIdx.y * 256 + threadIdx.x;
     int t = tok[r];
@@ -66,16 +67,59 @@ __global__ void __launch_bounds__(256) embed_kernel(const WT* embed, const int32
 // Greedy acceptance (Sec. 2.1): drafts = rows[1..gamma], z = target argmax of
 // rows[0..gamma].  a = longest prefix with drafts[i] == z[i]; the new tokens
 // are drafts[0..a-1] followed by z[a], which becomes the pending rows[0].
-// result = {a, a + 1, tokens[0..a]}.
-__global__ void accept_kernel(int32_t* rows, const int32_t* z, int gamma, int32_t* result) {
+// After a dynamic-exit draft only the n_drafted drafts that were produced are
+// compared (the pass still scored gamma + 1 rows; the rest are ignored).
+// result = {a, drafts compared, tokens[0..a]}.
+__global__ void accept_kernel(int32_t* rows, const int32_t* z, int gamma, const int32_t* n_drafted,
+                              int32_t* result) {
     if (threadIdx.x != 0) return;
+    const int g = n_drafted ? min(gamma, *n_drafted) : gamma;
     int a = 0;
-    while (a < gamma && rows[1 + a] == z[a]) ++a;
+    while (a < g && rows[1 + a] == z[a]) ++a;
     result[0] = a;
-    result[1] = a + 1;
+    result[1] = g;
     for (int i = 0; i < a; ++i) result[2 + i] = rows[1 + i];
     result[2 + a] = z[a];
     rows[0] = z[a];
+}
+
+// Dynamic drafting exit (Sec. 3.5): the confidence of draft pass t's token is
+// its softmax probability, 1 / sum_i exp(l_i - l_max), over the pass's logits
+// (row 0); l_max is the logit of the argmax token the LM head wrote.  Each of
+// kTop1Ctas CTAs sums exp(l_i - l_max) over a fixed slice of the vocabulary
+// in a fixed order; the last CTA to finish adds the slices in slice order, so
+// the value is the same in every run.  It records the confidence, counts the
+// pass as drafted, and raises the stop flag below tau, which makes the later
+// draft passes of the step return at once.
+constexpr int kTop1Ctas = 64;
+constexpr int kTop1Threads = 256;
+__global__ void __launch_bounds__(kTop1Threads) top1_kernel(const float* logits, int vocab, const int32_t* token,
+                                                            float tau, int t, int* stop, int* n_drafted,
+                                                            float* conf, float* part, int* ticket) {
+    if (*stop) return;
+    __shared__ float red[kTop1Threads / 32 + 1];
+    __shared__ int last;
+    const float lmax = logits[*token];
+    const int per = (vocab + kTop1Ctas - 1) / kTop1Ctas;
+    const int lo = blockIdx.x * per, hi = min(vocab, lo + per);
+    float s = 0.f;
+    for (int i = lo + (int)threadIdx.x; i < hi; i += kTop1Threads) s += expf(logits[i] - lmax);
+    s = block_sum<kTop1Threads / 32>(s, red);
+    if (threadIdx.x == 0) {
+        part[blockIdx.x] = s;
+        __threadfence();
+        last = atomicAdd(ticket, 1) == kTop1Ctas - 1;
+    }
+    __syncthreads();
+    if (!last || threadIdx.x != 0) return;
+    __threadfence();
+    float S = 0.f;
+    for (int c = 0; c < kTop1Ctas; ++c) S += __ldcg(&part[c]);
+    const float p1 = 1.f / S;
+    conf[t] = p1;
+    *n_drafted = t + 1;
+    if (p1 < tau) *stop = 1;
+    *ticket = 0;
 }
 
 // TPT stage, Eq. 4 inputs: row b of a batch is overall row q = row0 + b, i.e.
@@ -116,7 +160,7 @@ static size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 struct Layout {
     size_t kv, rope, x, ss, xg, qkv, attn_out, act, attn_part, gemv_part, counters, logits, amax_val,
         amax_idx, tok, hist, hist_snap, hist_idx, sims, mask, obj, wts, select, chain_ctr, best, tpt_masks,
-        tpt_tok, tpt_info, tpt_out, total;
+        tpt_tok, tpt_info, tpt_out, dyn, total;
     int n_chunks_max;
     size_t gemv_part_floats;
     int counters_n;
@@ -203,6 +247,8 @@ static Layout make_layout(const ks_config* c) {
     L.tpt_tok = take(sizeof(int32_t) * (KS_TPT_MAX_CANDIDATES + 1) * (size_t)L.hist_slots * R);
     L.tpt_info = take(sizeof(int32_t) * 4);
     L.tpt_out = take(sizeof(double) * (KS_TPT_MAX_CANDIDATES + 1));
+    // dynamic exit: confidence[max_rows] | slice sums[kTop1Ctas] | ticket
+    L.dyn = take(sizeof(float) * ((size_t)R + kTop1Ctas) + sizeof(int));
     L.total = off;
     return L;
 }
@@ -245,6 +291,13 @@ struct ks_model {
     int32_t* tpt_tok;
     int32_t* tpt_info;
     double* tpt_out;
+    float* conf;              // dynamic exit: confidence of each draft pass of the step
+    float* top1_part;         // dynamic exit: slice sums
+    int* top1_ticket;
+    int* stop;                // dynamic exit: set once a draft token is below tau_conf
+    int* n_drafted;           // dynamic exit: draft passes of the step that ran
+    bool last_dynamic = false;
+    int last_scored = 0;      // drafts compared by the last verify
     int chain_parity = 0;
     double* obj_dev;
     int* wts_dev;
@@ -333,7 +386,7 @@ static void* vcache(ks_model* m, int layer) {
 // sublayers must run).  argmax: device int32[R] for the LM head argmax, or
 // null to skip the LM head.
 static ks_status forward(ks_model* m, const int32_t* tok, int R, int p0, const uint8_t* mask,
-                         int capture_slot, int32_t* argmax) {
+                         int capture_slot, int32_t* argmax, const int* stop = nullptr) {
     const ks_config& c = m->cfg;
     const int d = c.d_model, hd = c.head_dim;
     const int nqkv = (c.n_q_heads + 2 * c.n_kv_heads) * hd;
@@ -387,15 +440,16 @@ static ks_status forward(ks_model* m, const int32_t* tok, int R, int p0, const u
         g.partial = m->gemv_part;
         g.counters = m->counters;
         g.err = m->err;
+        g.stop = stop;
     };
     KS_TRY(launch(m, K_EMBED, [&]() -> cudaError_t {
         if (bf)
             embed_kernel<__nv_bfloat16><<<dim3(R, (d + 255) / 256), 256, 0, s>>>(
                 reinterpret_cast<const __nv_bfloat16*>(m->embed), tok, d, c.vocab, m->x, cap_ptr(0), m->ss, m->xg,
-                reinterpret_cast<const __nv_bfloat16*>(next_gain(0)));
+                reinterpret_cast<const __nv_bfloat16*>(next_gain(0)), stop);
         else
             embed_kernel<float><<<dim3(R, (d + 255) / 256), 256, 0, s>>>(reinterpret_cast<const float*>(m->embed), tok, d, c.vocab, m->x,
-                                                  cap_ptr(0), m->ss, nullptr, nullptr);
+                                                  cap_ptr(0), m->ss, nullptr, nullptr, stop);
         return cudaGetLastError();
     }, "embed"));
 
@@ -411,6 +465,7 @@ static ks_status forward(ks_model* m, const int32_t* tok, int R, int p0, const u
         at.eps = c.rms_eps;
         at.part = m->attn_part; at.n_chunks_max = m->lay.n_chunks_max;
         at.out = m->attn_out; at.out_ld = c.n_q_heads * hd;
+        at.stop = stop;
         KS_TRY(launch(m, K_ATTN, [&] { return launch_attention(dt, at, s); }, "attention"));
         KS_TRY(launch(m, K_MERGE, [&] { return launch_attn_merge(dt, at, s); }, "attention merge"));
         return KS_OK;
@@ -444,6 +499,7 @@ static ks_status forward(ks_model* m, const int32_t* tok, int R, int p0, const u
         ca.capture = capture_slot >= 0 ? hist_plane(m, 0) + (size_t)capture_slot * c.max_rows * d : nullptr;
         ca.capture_plane = (long long)m->lay.hist_slots * c.max_rows * d;
         ca.err = m->err;
+        ca.stop = stop;
         int nph = 0, klass = K_CHAIN;
         double bytes = 0.0;
         auto flush = [&]() -> ks_status {
@@ -682,6 +738,11 @@ ks_status ks_model_create(const ks_config* cfg, const ks_weights* w, void* works
     m->tpt_tok = reinterpret_cast<int32_t*>(b + lay.tpt_tok);
     m->tpt_info = reinterpret_cast<int32_t*>(b + lay.tpt_info);
     m->tpt_out = reinterpret_cast<double*>(b + lay.tpt_out);
+    m->conf = reinterpret_cast<float*>(b + lay.dyn);
+    m->top1_part = m->conf + cfg->max_rows;
+    m->top1_ticket = reinterpret_cast<int*>(m->top1_part + kTop1Ctas);
+    m->stop = m->rows + (3 * cfg->max_rows + 5);        // spare words of the token block
+    m->n_drafted = m->rows + (3 * cfg->max_rows + 6);
     m->obj_dev = reinterpret_cast<double*>(b + lay.obj);
     m->wts_dev = reinterpret_cast<int*>(b + lay.wts);
     m->select = b + lay.select;
@@ -753,6 +814,8 @@ ks_status ks_model_create(const ks_config* cfg, const ks_weights* w, void* works
     if (e != cudaSuccess) return fail(e, "counter reset");
     e = cudaMemsetAsync(b + lay.tok, 0, sizeof(int) * ((size_t)3 * R + 8 + cfg->max_seq), m->stream);  // incl. err
     if (e != cudaSuccess) return fail(e, "token reset");
+    e = cudaMemsetAsync(b + lay.dyn, 0, sizeof(float) * ((size_t)R + kTop1Ctas) + sizeof(int), m->stream);
+    if (e != cudaSuccess) return fail(e, "dynamic-exit reset");
     e = cudaStreamSynchronize(m->stream);
     if (e != cudaSuccess) return fail(e, "create sync");
     *out = m;
@@ -774,6 +837,7 @@ ks_status ks_model_destroy(ks_model* m) {
 // the prompt's final chunk (lastlen rows captured in slot 0).
 static void reset_history(ks_model* m, int lastlen) {
     m->last_gamma = -1;
+    m->last_dynamic = false;
     std::fill(m->slot_cnt.begin(), m->slot_cnt.end(), 0);
     const int init = std::min(m->cfg.hist_init_rows, lastlen);
     m->slot_off[0] = lastlen - init;
@@ -889,12 +953,60 @@ ks_status ks_draft(ks_model* m, const uint8_t* mask, int32_t gamma, int32_t* dra
     for (int t = 0; t < gamma; ++t)
         KS_TRY(forward(m, m->rows + t, 1, m->p + t, mask, -1, m->rows + t + 1));
     m->last_gamma = gamma;
+    m->last_dynamic = false;
     if (draft_tokens) {
         KS_CUDA(cudaMemcpyAsync(m->h_buf, m->rows + 1, sizeof(int32_t) * gamma, cudaMemcpyDeviceToHost, m->stream),
                 "draft download");
         m->d2h += sizeof(int32_t) * gamma;
         KS_TRY(sync(m, "ks_draft"));
         std::memcpy(draft_tokens, m->h_buf, sizeof(int32_t) * gamma);
+    }
+    return KS_OK;
+}
+
+ks_status ks_draft_dynamic(ks_model* m, const uint8_t* mask, int32_t gamma, float tau_conf, int32_t* n_drafted,
+                           float* confidence, int32_t* draft_tokens) {
+    if (!m || !mask) {
+        set_error("ks_draft_dynamic: null argument");
+        return KS_ERR_INVALID_ARG;
+    }
+    if (!m->have_seq) {
+        set_error("ks_draft_dynamic: no sequence (call ks_prefill first)");
+        return KS_ERR_STATE;
+    }
+    if (gamma < 1 || gamma >= m->cfg.max_rows || !(tau_conf >= 0.f) || !std::isfinite(tau_conf)) {
+        set_error("ks_draft_dynamic: gamma must be in [1, max_rows) and tau_conf finite and >= 0");
+        return KS_ERR_INVALID_ARG;
+    }
+    if (m->p + gamma + 1 > m->cfg.max_seq) {
+        set_error("ks_draft_dynamic: KV capacity exceeded");
+        return KS_ERR_CAPACITY;
+    }
+    cudaStream_t s = m->stream;
+    // a new step: no pass has run and none has stopped (stop and n_drafted are adjacent)
+    KS_CUDA(cudaMemsetAsync(m->stop, 0, 2 * sizeof(int), s), "dynamic-exit reset");
+    for (int t = 0; t < gamma; ++t) {
+        KS_TRY(forward(m, m->rows + t, 1, m->p + t, mask, -1, m->rows + t + 1, m->stop));
+        KS_TRY(launch(m, K_ACCEPT, [&]() -> cudaError_t {
+            top1_kernel<<<kTop1Ctas, kTop1Threads, 0, s>>>(m->logits, m->cfg.vocab, m->rows + t + 1, tau_conf, t,
+                                                           m->stop, m->n_drafted, m->conf, m->top1_part,
+                                                           m->top1_ticket);
+            return cudaGetLastError();
+        }, "draft confidence"));
+    }
+    m->last_gamma = gamma;
+    m->last_dynamic = true;
+    if (n_drafted || confidence || draft_tokens) {
+        int32_t* hb = m->h_buf;   // tokens [0, 16), count [16], confidences [32, 48)
+        KS_CUDA(cudaMemcpyAsync(hb, m->rows + 1, sizeof(int32_t) * gamma, cudaMemcpyDeviceToHost, s), "draft download");
+        KS_CUDA(cudaMemcpyAsync(hb + 16, m->n_drafted, sizeof(int32_t), cudaMemcpyDeviceToHost, s), "draft download");
+        KS_CUDA(cudaMemcpyAsync(hb + 32, m->conf, sizeof(float) * gamma, cudaMemcpyDeviceToHost, s), "draft download");
+        m->d2h += sizeof(int32_t) * (gamma + 1) + sizeof(float) * gamma;
+        KS_TRY(sync(m, "ks_draft_dynamic"));
+        const int n = hb[16];
+        if (n_drafted) *n_drafted = n;
+        if (draft_tokens) std::memcpy(draft_tokens, hb, sizeof(int32_t) * n);
+        if (confidence) std::memcpy(confidence, hb + 32, sizeof(float) * n);
     }
     return KS_OK;
 }
@@ -936,7 +1048,9 @@ ks_status ks_verify(ks_model* m, const int32_t* draft_tokens, int32_t gamma, int
     const int slot = m->hist_next;
     KS_TRY(forward(m, m->rows, R, m->p, nullptr, slot, m->target));
     KS_TRY(launch(m, K_ACCEPT, [&]() -> cudaError_t {
-        accept_kernel<<<1, 32, 0, m->stream>>>(m->rows, m->target, gamma, m->result);
+        accept_kernel<<<1, 32, 0, m->stream>>>(m->rows, m->target, gamma,
+                                               (m->last_dynamic && !draft_tokens) ? m->n_drafted : nullptr,
+                                               m->result);
         return cudaGetLastError();
     }, "accept"));
     int32_t* hb = m->h_buf + m->cfg.max_seq + 2 * m->cfg.max_rows;
@@ -945,7 +1059,8 @@ ks_status ks_verify(ks_model* m, const int32_t* draft_tokens, int32_t gamma, int
     m->d2h += sizeof(int32_t) * (gamma + 3);
     KS_TRY(sync(m, "ks_verify"));
     const int a = hb[0];
-    if (a < 0 || a > gamma) {
+    const int scored = hb[1];
+    if (a < 0 || scored < 0 || scored > gamma || a > scored) {
         set_error("ks_verify: corrupt acceptance result");
         return KS_ERR_CUDA;
     }
@@ -960,6 +1075,8 @@ ks_status ks_verify(ks_model* m, const int32_t* draft_tokens, int32_t gamma, int
     // keep hist_steps entries: drop the entry the next verify will overwrite
     m->slot_cnt[m->hist_next] = 0;
     m->last_gamma = -1;
+    m->last_dynamic = false;
+    m->last_scored = scored;
     return KS_OK;
 }
 
@@ -989,6 +1106,7 @@ ks_status ks_decode_greedy(ks_model* m, int32_t n_tokens, int32_t* out) {
     m->p += n_tokens - 1;
     m->pending = out[n_tokens - 1];
     m->last_gamma = -1;
+    m->last_dynamic = false;
     return KS_OK;
 }
 
@@ -1031,6 +1149,7 @@ static ks_status lm_head_rows(ks_model* m, int R, int32_t* tokens) {
         ca.logits = m->logits; ca.best = m->best; ca.tokens = tokens;
         ca.capture = nullptr;
         ca.err = m->err;
+        ca.stop = nullptr;
         ca.n_phases = 1;
         ca.code[0] = (uint16_t)(4 * L);
         ca.gain[0] = nullptr;
@@ -1208,6 +1327,10 @@ ks_status ks_generate_speculative(ks_model* m, const ks_spec_params* prm, int32_
         set_error("ks_generate_speculative: bad parameters");
         return KS_ERR_INVALID_ARG;
     }
+    if (!(prm->tau_conf >= 0.0) || !std::isfinite(prm->tau_conf)) {
+        set_error("ks_generate_speculative: tau_conf must be finite and >= 0");
+        return KS_ERR_INVALID_ARG;
+    }
     if (prm->policy != 0 && !latency_ok(prm->latency, nsub)) {
         set_error("ks_generate_speculative: bad latency model");
         return KS_ERR_INVALID_ARG;
@@ -1255,12 +1378,15 @@ ks_status ks_generate_speculative(ks_model* m, const ks_spec_params* prm, int32_
             set_error("ks_generate_speculative: KV capacity exhausted");
             return KS_ERR_CAPACITY;
         }
-        KS_TRY(ks_draft(m, mask.data(), g, nullptr));
+        if (prm->tau_conf > 0.0)
+            KS_TRY(ks_draft_dynamic(m, mask.data(), g, (float)prm->tau_conf, nullptr, nullptr, nullptr));
+        else
+            KS_TRY(ks_draft(m, mask.data(), g, nullptr));
         int32_t a = 0, no = 0;
         KS_TRY(ks_verify(m, nullptr, g, &a, toks.data(), &no));
         if (accepted_per_step) accepted_per_step[st.steps] = a;
         st.steps++;
-        st.drafted += g;
+        st.drafted += m->last_scored;
         st.accepted += a;
         for (int i = 0; i < no && n < n_tokens; ++i) out[n++] = toks[i];
     }

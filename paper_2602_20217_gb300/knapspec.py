@@ -47,7 +47,8 @@ class KsLatency(C.Structure):
 class KsSpecParams(C.Structure):
     _fields_ = [("gamma", C.c_int32), ("policy", C.c_int32), ("mask", C.POINTER(C.c_uint8)),
                 ("latency", KsLatency), ("budget_frac", C.c_double), ("resolve_every", C.c_int32),
-                ("max_steps", C.c_int32), ("tpt_candidates", C.c_int32), ("tpt_max_gamma", C.c_int32)]
+                ("max_steps", C.c_int32), ("tpt_candidates", C.c_int32), ("tpt_max_gamma", C.c_int32),
+                ("tau_conf", C.c_double)]
 
 
 class KsSpecStats(C.Structure):
@@ -71,6 +72,8 @@ _SIGS = {
     "ks_prefill": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.POINTER(C.c_int32)]),
     "ks_rewind": (C.c_int, [C.c_void_p, C.POINTER(C.c_int32)]),
     "ks_draft": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p]),
+    "ks_draft_dynamic": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.c_float, C.c_void_p, C.c_void_p,
+                                   C.c_void_p]),
     "ks_verify": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.POINTER(C.c_int32), C.c_void_p,
                             C.POINTER(C.c_int32)]),
     "ks_decode_greedy": (C.c_int, [C.c_void_p, C.c_int32, C.c_void_p]),
@@ -207,6 +210,22 @@ def ks_draft(h: int, mask, gamma: int, want_tokens: bool = True):
     out = np.zeros(gamma, np.int32) if want_tokens else None
     check(load().ks_draft(h, m.ctypes.data, gamma, out.ctypes.data if want_tokens else None), "ks_draft")
     return out
+
+
+def ks_draft_dynamic(h: int, mask, gamma: int, tau_conf: float, want_outputs: bool = True):
+    """Drafts with the dynamic exit: (n_drafted, confidences[n], tokens[n]), or
+    None without waiting when want_outputs is False."""
+    m = np.ascontiguousarray(mask, dtype=np.uint8)
+    if not want_outputs:
+        check(load().ks_draft_dynamic(h, m.ctypes.data, gamma, float(tau_conf), None, None, None),
+              "ks_draft_dynamic")
+        return None
+    n = C.c_int32()
+    conf = np.zeros(gamma, np.float32)
+    toks = np.zeros(gamma, np.int32)
+    check(load().ks_draft_dynamic(h, m.ctypes.data, gamma, float(tau_conf), C.byref(n), conf.ctypes.data,
+                                  toks.ctypes.data), "ks_draft_dynamic")
+    return n.value, conf[: n.value], toks[: n.value]
 
 
 def ks_verify(h: int, draft_tokens, gamma: int):

@@ -38,6 +38,10 @@ class Model:
     def draft(self, mask, gamma: int):
         return ks.ks_draft(self.h, mask, gamma)
 
+    def draft_dynamic(self, mask, gamma: int, tau_conf: float):
+        """Drafts with the dynamic exit (Sec. 3.5): (n_drafted, confidences, tokens)."""
+        return ks.ks_draft_dynamic(self.h, mask, gamma, tau_conf)
+
     def verify(self, drafts, gamma: int):
         return ks.ks_verify(self.h, drafts, gamma)
 
@@ -48,25 +52,28 @@ class Model:
         return ks.ks_model_position(self.h)
 
     def generate(self, n_tokens: int, gamma: int, mask=None, latency=None, budget_frac: float = 0.5,
-                 resolve_every: int = 64, max_steps: int = 0, tpt=None):
+                 resolve_every: int = 64, max_steps: int = 0, tpt=None, tau_conf: float = 0.0):
         """Speculative decoding: a fixed mask (policy 0), the knapsack policy
         (policy 1, latency given) or the TPT stage (policy 2, latency and
-        tpt = (n_candidates, max_gamma) given)."""
+        tpt = (n_candidates, max_gamma) given); tau_conf > 0 adds the dynamic
+        drafting exit."""
         n = self.shape.n_sublayers
         keep = []
         if latency is None:
             m = np.ascontiguousarray(mask if mask is not None else np.ones(n), dtype=np.uint8)
             keep.append(m)
             lat, _ = ks.latency(0, 1.0, 0.0, 1.0)
-            p = ks.KsSpecParams(gamma, 0, m.ctypes.data_as(ks.C.POINTER(ks.C.c_uint8)), lat, 0.0, 1, max_steps)
+            p = ks.KsSpecParams(gamma, 0, m.ctypes.data_as(ks.C.POINTER(ks.C.c_uint8)), lat, 0.0, 1, max_steps,
+                                0, 0, float(tau_conf))
         else:
             lat, u = latency
             keep.append(u)
             if tpt is None:
-                p = ks.KsSpecParams(gamma, 1, None, lat, float(budget_frac), int(resolve_every), max_steps)
+                p = ks.KsSpecParams(gamma, 1, None, lat, float(budget_frac), int(resolve_every), max_steps,
+                                    0, 0, float(tau_conf))
             else:
                 p = ks.KsSpecParams(gamma, 2, None, lat, 0.0, int(resolve_every), max_steps,
-                                    int(tpt[0]), int(tpt[1]))
+                                    int(tpt[0]), int(tpt[1]), float(tau_conf))
         return ks.ks_generate_speculative(self.h, p, n_tokens)
 
     def select_tpt(self, latency, n_candidates: int, max_gamma: int):

@@ -89,6 +89,7 @@ def test_error_paths_touch_no_device(lib):
     a, n = C.c_int32(), C.c_int32()
     assert lib.ks_prefill(None, out.ctypes.data, 4, C.byref(a)) == ks.KS_ERR_INVALID_ARG
     assert lib.ks_draft(None, out.ctypes.data, 4, None) == ks.KS_ERR_INVALID_ARG
+    assert lib.ks_draft_dynamic(None, out.ctypes.data, 4, 0.7, None, None, None) == ks.KS_ERR_INVALID_ARG
     assert lib.ks_verify(None, None, 4, C.byref(a), out.ctypes.data, C.byref(n)) == ks.KS_ERR_INVALID_ARG
     assert lib.ks_decode_greedy(None, 4, out.ctypes.data) == ks.KS_ERR_INVALID_ARG
     assert lib.ks_model_destroy(None) == ks.KS_ERR_INVALID_ARG
