@@ -168,6 +168,40 @@ ks_status ks_draft(ks_model* m, const uint8_t* mask, int32_t gamma, int32_t* dra
 ks_status ks_draft_dynamic(ks_model* m, const uint8_t* mask, int32_t gamma, float tau_conf, int32_t* n_drafted,
                            float* confidence, int32_t* draft_tokens);
 
+/* Sampling mode (Sec. 2.1, sampling branch; the Sec. 4 experiments use
+ * temperature 0.7, top_k 50, top_p 0.95).  A distribution is the row's logits
+ * divided by the temperature, cut to the top_k largest (ties: lower id first;
+ * top_k above 64 is taken as 64), softmaxed, cut to the shortest prefix in
+ * descending probability whose cumulative probability reaches top_p, and
+ * renormalised.  Uniform numbers are Philox4x64-10 (Salmon et al., SC 2011)
+ * with key (seed, 0) and counter (step, row, purpose, 0): purpose 0 the draft
+ * sample of position row, 1 the acceptance test of draft row, 2 the step's
+ * residual or bonus sample; u = (first output word >> 40) / 2^24. */
+typedef struct {
+    float temperature;       /* > 0 (0 in ks_spec_params: greedy decoding)   */
+    int32_t top_k;           /* >= 1                                          */
+    float top_p;             /* (0, 1]                                        */
+    uint64_t seed;
+} ks_sampling;
+
+/* a1, sampling: gamma draft tokens of f^(S), each drawn from its draft
+ * distribution q_t with the uniform of (step, t, 0); the q_t stay on the
+ * device for ks_verify_sample.  draft_tokens: host int32[gamma] or NULL (then
+ * no synchronisation). */
+ks_status ks_draft_sample(ks_model* m, const uint8_t* mask, int32_t gamma, const ks_sampling* s, uint64_t step,
+                          int32_t* draft_tokens);
+
+/* a2 + a3, sampling (Sec. 2.1): score [pending, drafts...] of the preceding
+ * ks_draft_sample (same gamma, same step and sampling parameters) with the
+ * full target, form the target distributions p_0..p_gamma, and accept draft t
+ * while u(step, t, 1) <= min(1, p_t(x_t) / q_t(x_t)).  At the first rejection
+ * the next token is drawn from norm(max(0, p_t - q_t)) (from p_t if that has
+ * no mass), after gamma acceptances from p_gamma, with u(step, 0, 2).  The
+ * tokens are distributed as samples of the target.  Outputs and commit as
+ * ks_verify.  Waits for the stream. */
+ks_status ks_verify_sample(ks_model* m, int32_t gamma, const ks_sampling* s, uint64_t step, int32_t* n_accepted,
+                           int32_t* out_tokens, int32_t* n_out);
+
 /* a2 + a3 (Sec. 2.1): score [pending, drafts...] (gamma + 1 rows at positions
  * p..p+gamma) with the full target in one pass, take the greedy argmax of
  * each row, accept the longest prefix of drafts equal to the target's
@@ -294,6 +328,9 @@ typedef struct {
     int32_t tpt_max_gamma;   /* policy 2: max_gamma of ks_select_tpt                        */
     double tau_conf;         /* > 0: dynamic drafting exit (ks_draft_dynamic) with this
                                 tau_conf; 0: every step drafts gamma tokens               */
+    ks_sampling sampling;    /* temperature > 0: sampling mode (ks_draft_sample /
+                                ks_verify_sample, step = the verify step index from 0);
+                                not combined with tau_conf                                 */
 } ks_spec_params;
 
 typedef struct {
@@ -323,6 +360,9 @@ ks_status ks_generate_speculative(ks_model* m, const ks_spec_params* params, int
  *        3: V cache, as 2;
  *        4: history ring states of the committed rows, float[2L+1][r][d], with
  *           count == r; count == 0 writes r itself (int32) to dst;
+ *        5: sampling draft distributions of positions [start, start + count):
+ *           per position int32 n, int32 ids[64], float probs[64] (first n used);
+ *        6: sampling target distributions of the last ks_verify_sample rows, as 5;
  * dst is host memory of `bytes` bytes; the call waits for the stream. */
 ks_status ks_debug_read(ks_model* m, int32_t what, int32_t layer, int32_t start, int32_t count,
                         void* dst, size_t bytes);

@@ -149,4 +149,32 @@ cudaError_t launch_cosine(const void* X, const void* Y, int dtype, int64_t n_pai
 // Last error text for ks_last_error (thread-local).
 void set_error(const char* fmt, ...);
 
+// ---------------------------------------------------------- sampling mode
+// Nucleus-filtered distributions (at most kSampleMaxK tokens per row) and the
+// Sec. 2.1 acceptance of sampling-mode speculative decoding (sample.cu).
+constexpr int kSampleMaxK = 64;
+struct FilterArgs {
+    const float* logits;    // [rows][ld] fp32
+    int ld, vocab;
+    float inv_t;            // 1 / temperature
+    int top_k;              // 1 .. kSampleMaxK (larger values are clamped)
+    float top_p;            // (0, 1]
+    int* ids;               // [slots][kSampleMaxK] support in descending probability
+    float* probs;           // [slots][kSampleMaxK] renormalised probabilities
+    int* n;                 // [slots] support sizes
+    int slot0;              // row r is stored at slot slot0 + r (a draft pass: its position t)
+    int32_t* token_out;     // draft pass: the drawn token goes here (null: no draw)
+    unsigned long long seed, step;
+};
+struct AcceptSampleArgs {
+    int32_t* rows;          // [gamma + 1]: pending, drafts; rows[0] <- the new pending token
+    int gamma;
+    const int* p_ids; const float* p_probs; const int* p_n;   // target rows 0..gamma
+    const int* q_ids; const float* q_probs; const int* q_n;   // draft positions 0..gamma-1
+    int32_t* result;        // {a, gamma, tokens[0..a]}
+    unsigned long long seed, step;
+};
+cudaError_t launch_filter(const FilterArgs& a, int rows, cudaStream_t s);
+cudaError_t launch_spec_accept(const AcceptSampleArgs& a, cudaStream_t s);
+
 }  // namespace ks

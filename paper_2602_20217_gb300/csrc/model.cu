@@ -160,7 +160,7 @@ static size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 struct Layout {
     size_t kv, rope, x, ss, xg, qkv, attn_out, act, attn_part, gemv_part, counters, logits, amax_val,
         amax_idx, tok, hist, hist_snap, hist_idx, sims, mask, obj, wts, select, chain_ctr, best, tpt_masks,
-        tpt_tok, tpt_info, tpt_out, dyn, total;
+        tpt_tok, tpt_info, tpt_out, dyn, samp, total;
     int n_chunks_max;
     size_t gemv_part_floats;
     int counters_n;
@@ -249,6 +249,8 @@ static Layout make_layout(const ks_config* c) {
     L.tpt_out = take(sizeof(double) * (KS_TPT_MAX_CANDIDATES + 1));
     // dynamic exit: confidence[max_rows] | slice sums[kTop1Ctas] | ticket
     L.dyn = take(sizeof(float) * ((size_t)R + kTop1Ctas) + sizeof(int));
+    // sampling: q and p distributions, [R][kSampleMaxK] ids and probs plus [R] sizes each
+    L.samp = take(2 * ((size_t)R * kSampleMaxK * (sizeof(int) + sizeof(float)) + sizeof(int) * R));
     L.total = off;
     return L;
 }
@@ -297,6 +299,9 @@ struct ks_model {
     int* stop;                // dynamic exit: set once a draft token is below tau_conf
     int* n_drafted;           // dynamic exit: draft passes of the step that ran
     bool last_dynamic = false;
+    bool last_sampled = false;   // the drafts on the device were sampled (ks_draft_sample)
+    int *q_ids, *q_n, *p_ids, *p_n;   // sampling mode: draft / target distributions [16][kSampleMaxK]
+    float *q_probs, *p_probs;
     int last_scored = 0;      // drafts compared by the last verify
     int chain_parity = 0;
     double* obj_dev;
@@ -743,6 +748,16 @@ ks_status ks_model_create(const ks_config* cfg, const ks_weights* w, void* works
     m->top1_ticket = reinterpret_cast<int*>(m->top1_part + kTop1Ctas);
     m->stop = m->rows + (3 * cfg->max_rows + 5);        // spare words of the token block
     m->n_drafted = m->rows + (3 * cfg->max_rows + 6);
+    {
+        char* sb = b + lay.samp;
+        const size_t RK = (size_t)cfg->max_rows * kSampleMaxK;
+        m->q_ids = reinterpret_cast<int*>(sb);
+        m->q_probs = reinterpret_cast<float*>(m->q_ids + RK);
+        m->q_n = reinterpret_cast<int*>(m->q_probs + RK);
+        m->p_ids = m->q_n + cfg->max_rows;
+        m->p_probs = reinterpret_cast<float*>(m->p_ids + RK);
+        m->p_n = reinterpret_cast<int*>(m->p_probs + RK);
+    }
     m->obj_dev = reinterpret_cast<double*>(b + lay.obj);
     m->wts_dev = reinterpret_cast<int*>(b + lay.wts);
     m->select = b + lay.select;
@@ -838,6 +853,7 @@ ks_status ks_model_destroy(ks_model* m) {
 static void reset_history(ks_model* m, int lastlen) {
     m->last_gamma = -1;
     m->last_dynamic = false;
+    m->last_sampled = false;
     std::fill(m->slot_cnt.begin(), m->slot_cnt.end(), 0);
     const int init = std::min(m->cfg.hist_init_rows, lastlen);
     m->slot_off[0] = lastlen - init;
@@ -954,6 +970,7 @@ ks_status ks_draft(ks_model* m, const uint8_t* mask, int32_t gamma, int32_t* dra
         KS_TRY(forward(m, m->rows + t, 1, m->p + t, mask, -1, m->rows + t + 1));
     m->last_gamma = gamma;
     m->last_dynamic = false;
+    m->last_sampled = false;
     if (draft_tokens) {
         KS_CUDA(cudaMemcpyAsync(m->h_buf, m->rows + 1, sizeof(int32_t) * gamma, cudaMemcpyDeviceToHost, m->stream),
                 "draft download");
@@ -996,6 +1013,7 @@ ks_status ks_draft_dynamic(ks_model* m, const uint8_t* mask, int32_t gamma, floa
     }
     m->last_gamma = gamma;
     m->last_dynamic = true;
+    m->last_sampled = false;
     if (n_drafted || confidence || draft_tokens) {
         int32_t* hb = m->h_buf;   // tokens [0, 16), count [16], confidences [32, 48)
         KS_CUDA(cudaMemcpyAsync(hb, m->rows + 1, sizeof(int32_t) * gamma, cudaMemcpyDeviceToHost, s), "draft download");
@@ -1011,8 +1029,11 @@ ks_status ks_draft_dynamic(ks_model* m, const uint8_t* mask, int32_t gamma, floa
     return KS_OK;
 }
 
-ks_status ks_verify(ks_model* m, const int32_t* draft_tokens, int32_t gamma, int32_t* n_accepted,
-                    int32_t* out_tokens, int32_t* n_out) {
+// a2 + a3; sp != null: the sampling branch of Sec. 2.1 over the drafts of
+// the preceding ks_draft_sample (filtered target rows, then the acceptance
+// with residual resampling), else greedy acceptance.
+static ks_status verify_impl(ks_model* m, const int32_t* draft_tokens, int32_t gamma, const ks_sampling* sp,
+                             unsigned long long step, int32_t* n_accepted, int32_t* out_tokens, int32_t* n_out) {
     if (!m || !n_accepted || !out_tokens || !n_out) {
         set_error("ks_verify: null argument");
         return KS_ERR_INVALID_ARG;
@@ -1047,12 +1068,27 @@ ks_status ks_verify(ks_model* m, const int32_t* draft_tokens, int32_t gamma, int
     const int R = gamma + 1;
     const int slot = m->hist_next;
     KS_TRY(forward(m, m->rows, R, m->p, nullptr, slot, m->target));
-    KS_TRY(launch(m, K_ACCEPT, [&]() -> cudaError_t {
-        accept_kernel<<<1, 32, 0, m->stream>>>(m->rows, m->target, gamma,
-                                               (m->last_dynamic && !draft_tokens) ? m->n_drafted : nullptr,
-                                               m->result);
-        return cudaGetLastError();
-    }, "accept"));
+    if (sp) {
+        FilterArgs f{};
+        f.logits = m->logits; f.ld = m->cfg.vocab; f.vocab = m->cfg.vocab;
+        f.inv_t = 1.f / sp->temperature; f.top_k = sp->top_k; f.top_p = sp->top_p;
+        f.ids = m->p_ids; f.probs = m->p_probs; f.n = m->p_n; f.slot0 = 0; f.token_out = nullptr;
+        f.seed = sp->seed; f.step = step;
+        KS_TRY(launch(m, K_ACCEPT, [&] { return launch_filter(f, R, m->stream); }, "target distributions"));
+        AcceptSampleArgs ac{};
+        ac.rows = m->rows; ac.gamma = gamma;
+        ac.p_ids = m->p_ids; ac.p_probs = m->p_probs; ac.p_n = m->p_n;
+        ac.q_ids = m->q_ids; ac.q_probs = m->q_probs; ac.q_n = m->q_n;
+        ac.result = m->result; ac.seed = sp->seed; ac.step = step;
+        KS_TRY(launch(m, K_ACCEPT, [&] { return launch_spec_accept(ac, m->stream); }, "sampling acceptance"));
+    } else {
+        KS_TRY(launch(m, K_ACCEPT, [&]() -> cudaError_t {
+            accept_kernel<<<1, 32, 0, m->stream>>>(m->rows, m->target, gamma,
+                                                   (m->last_dynamic && !draft_tokens) ? m->n_drafted : nullptr,
+                                                   m->result);
+            return cudaGetLastError();
+        }, "accept"));
+    }
     int32_t* hb = m->h_buf + m->cfg.max_seq + 2 * m->cfg.max_rows;
     KS_CUDA(cudaMemcpyAsync(hb, m->result, sizeof(int32_t) * (gamma + 3), cudaMemcpyDeviceToHost, m->stream),
             "result download");
@@ -1076,8 +1112,81 @@ ks_status ks_verify(ks_model* m, const int32_t* draft_tokens, int32_t gamma, int
     m->slot_cnt[m->hist_next] = 0;
     m->last_gamma = -1;
     m->last_dynamic = false;
+    m->last_sampled = false;
     m->last_scored = scored;
     return KS_OK;
+}
+
+ks_status ks_verify(ks_model* m, const int32_t* draft_tokens, int32_t gamma, int32_t* n_accepted,
+                    int32_t* out_tokens, int32_t* n_out) {
+    if (m && !draft_tokens && m->last_sampled) {
+        set_error("ks_verify: the preceding drafts were sampled (use ks_verify_sample)");
+        return KS_ERR_STATE;
+    }
+    return verify_impl(m, draft_tokens, gamma, nullptr, 0ull, n_accepted, out_tokens, n_out);
+}
+
+static bool sampling_ok(const ks_sampling* sp) {
+    return sp && sp->temperature > 0.f && std::isfinite(sp->temperature) && sp->top_k >= 1 &&
+           sp->top_p > 0.f && sp->top_p <= 1.f;
+}
+
+ks_status ks_draft_sample(ks_model* m, const uint8_t* mask, int32_t gamma, const ks_sampling* sp, uint64_t step,
+                          int32_t* draft_tokens) {
+    if (!m || !mask || !sp) {
+        set_error("ks_draft_sample: null argument");
+        return KS_ERR_INVALID_ARG;
+    }
+    if (!m->have_seq) {
+        set_error("ks_draft_sample: no sequence (call ks_prefill first)");
+        return KS_ERR_STATE;
+    }
+    if (gamma < 1 || gamma >= m->cfg.max_rows || !sampling_ok(sp)) {
+        set_error("ks_draft_sample: gamma must be in [1, max_rows); temperature > 0, top_k >= 1, 0 < top_p <= 1");
+        return KS_ERR_INVALID_ARG;
+    }
+    if (m->p + gamma + 1 > m->cfg.max_seq) {
+        set_error("ks_draft_sample: KV capacity exceeded");
+        return KS_ERR_CAPACITY;
+    }
+    for (int t = 0; t < gamma; ++t) {
+        KS_TRY(forward(m, m->rows + t, 1, m->p + t, mask, -1, m->rows + t + 1));
+        FilterArgs f{};
+        f.logits = m->logits; f.ld = m->cfg.vocab; f.vocab = m->cfg.vocab;
+        f.inv_t = 1.f / sp->temperature; f.top_k = sp->top_k; f.top_p = sp->top_p;
+        f.ids = m->q_ids; f.probs = m->q_probs; f.n = m->q_n; f.slot0 = t;
+        f.token_out = m->rows + t + 1;   // replaces the LM head's argmax
+        f.seed = sp->seed; f.step = step;
+        KS_TRY(launch(m, K_ACCEPT, [&] { return launch_filter(f, 1, m->stream); }, "draft sample"));
+    }
+    m->last_gamma = gamma;
+    m->last_dynamic = false;
+    m->last_sampled = true;
+    if (draft_tokens) {
+        KS_CUDA(cudaMemcpyAsync(m->h_buf, m->rows + 1, sizeof(int32_t) * gamma, cudaMemcpyDeviceToHost, m->stream),
+                "draft download");
+        m->d2h += sizeof(int32_t) * gamma;
+        KS_TRY(sync(m, "ks_draft_sample"));
+        std::memcpy(draft_tokens, m->h_buf, sizeof(int32_t) * gamma);
+    }
+    return KS_OK;
+}
+
+ks_status ks_verify_sample(ks_model* m, int32_t gamma, const ks_sampling* sp, uint64_t step, int32_t* n_accepted,
+                           int32_t* out_tokens, int32_t* n_out) {
+    if (!m || !sp) {
+        set_error("ks_verify_sample: null argument");
+        return KS_ERR_INVALID_ARG;
+    }
+    if (!sampling_ok(sp)) {
+        set_error("ks_verify_sample: temperature > 0, top_k >= 1, 0 < top_p <= 1");
+        return KS_ERR_INVALID_ARG;
+    }
+    if (!m->last_sampled || m->last_gamma != gamma) {
+        set_error("ks_verify_sample: no preceding ks_draft_sample with this gamma");
+        return KS_ERR_STATE;
+    }
+    return verify_impl(m, nullptr, gamma, sp, step, n_accepted, out_tokens, n_out);
 }
 
 ks_status ks_decode_greedy(ks_model* m, int32_t n_tokens, int32_t* out) {
@@ -1107,6 +1216,7 @@ ks_status ks_decode_greedy(ks_model* m, int32_t n_tokens, int32_t* out) {
     m->pending = out[n_tokens - 1];
     m->last_gamma = -1;
     m->last_dynamic = false;
+    m->last_sampled = false;
     return KS_OK;
 }
 
@@ -1331,6 +1441,12 @@ ks_status ks_generate_speculative(ks_model* m, const ks_spec_params* prm, int32_
         set_error("ks_generate_speculative: tau_conf must be finite and >= 0");
         return KS_ERR_INVALID_ARG;
     }
+    const bool sampling = prm->sampling.temperature != 0.f;
+    if (sampling && (!sampling_ok(&prm->sampling) || prm->tau_conf > 0.0)) {
+        set_error("ks_generate_speculative: sampling needs temperature > 0, top_k >= 1, 0 < top_p <= 1 "
+                  "and no dynamic exit");
+        return KS_ERR_INVALID_ARG;
+    }
     if (prm->policy != 0 && !latency_ok(prm->latency, nsub)) {
         set_error("ks_generate_speculative: bad latency model");
         return KS_ERR_INVALID_ARG;
@@ -1378,12 +1494,18 @@ ks_status ks_generate_speculative(ks_model* m, const ks_spec_params* prm, int32_
             set_error("ks_generate_speculative: KV capacity exhausted");
             return KS_ERR_CAPACITY;
         }
-        if (prm->tau_conf > 0.0)
-            KS_TRY(ks_draft_dynamic(m, mask.data(), g, (float)prm->tau_conf, nullptr, nullptr, nullptr));
-        else
-            KS_TRY(ks_draft(m, mask.data(), g, nullptr));
         int32_t a = 0, no = 0;
-        KS_TRY(ks_verify(m, nullptr, g, &a, toks.data(), &no));
+        if (sampling) {
+            const unsigned long long step = (unsigned long long)st.steps;
+            KS_TRY(ks_draft_sample(m, mask.data(), g, &prm->sampling, step, nullptr));
+            KS_TRY(ks_verify_sample(m, g, &prm->sampling, step, &a, toks.data(), &no));
+        } else {
+            if (prm->tau_conf > 0.0)
+                KS_TRY(ks_draft_dynamic(m, mask.data(), g, (float)prm->tau_conf, nullptr, nullptr, nullptr));
+            else
+                KS_TRY(ks_draft(m, mask.data(), g, nullptr));
+            KS_TRY(ks_verify(m, nullptr, g, &a, toks.data(), &no));
+        }
         if (accepted_per_step) accepted_per_step[st.steps] = a;
         st.steps++;
         st.drafted += m->last_scored;
@@ -1421,6 +1543,30 @@ ks_status ks_debug_read(ks_model* m, int32_t what, int32_t layer, int32_t start,
                                   c.n_kv_heads, cudaMemcpyDeviceToHost, s),
                 "debug kv read");
         return sync(m, "debug kv read");
+    }
+    if (what == 5 || what == 6) {
+        // sampling distributions: per slot n, ids[kSampleMaxK], probs[kSampleMaxK] (int32, int32, float)
+        if (start < 0 || count < 1 || start + count > c.max_rows ||
+            bytes < sizeof(int32_t) * (size_t)count * (1 + 2 * kSampleMaxK))
+            return KS_ERR_INVALID_ARG;
+        const int* ids = what == 5 ? m->q_ids : m->p_ids;
+        const float* pr = what == 5 ? m->q_probs : m->p_probs;
+        const int* n = what == 5 ? m->q_n : m->p_n;
+        std::vector<int32_t> hn(count), hi((size_t)count * kSampleMaxK);
+        std::vector<float> hp((size_t)count * kSampleMaxK);
+        KS_CUDA(cudaMemcpy(hn.data(), n + start, sizeof(int32_t) * count, cudaMemcpyDeviceToHost), "debug read");
+        KS_CUDA(cudaMemcpy(hi.data(), ids + (size_t)start * kSampleMaxK, sizeof(int32_t) * hi.size(),
+                           cudaMemcpyDeviceToHost), "debug read");
+        KS_CUDA(cudaMemcpy(hp.data(), pr + (size_t)start * kSampleMaxK, sizeof(float) * hp.size(),
+                           cudaMemcpyDeviceToHost), "debug read");
+        int32_t* out = reinterpret_cast<int32_t*>(dst);
+        for (int r = 0; r < count; ++r) {
+            int32_t* o = out + (size_t)r * (1 + 2 * kSampleMaxK);
+            o[0] = hn[r];
+            std::memcpy(o + 1, hi.data() + (size_t)r * kSampleMaxK, sizeof(int32_t) * kSampleMaxK);
+            std::memcpy(o + 1 + kSampleMaxK, hp.data() + (size_t)r * kSampleMaxK, sizeof(float) * kSampleMaxK);
+        }
+        return KS_OK;
     }
     if (what == 4) {
         std::vector<int32_t> idx(m->lay.hist_slots * c.max_rows);

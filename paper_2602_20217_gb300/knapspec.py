@@ -44,11 +44,15 @@ class KsLatency(C.Structure):
                 ("units", C.POINTER(C.c_int32))]
 
 
+class KsSampling(C.Structure):
+    _fields_ = [("temperature", C.c_float), ("top_k", C.c_int32), ("top_p", C.c_float), ("seed", C.c_uint64)]
+
+
 class KsSpecParams(C.Structure):
     _fields_ = [("gamma", C.c_int32), ("policy", C.c_int32), ("mask", C.POINTER(C.c_uint8)),
                 ("latency", KsLatency), ("budget_frac", C.c_double), ("resolve_every", C.c_int32),
                 ("max_steps", C.c_int32), ("tpt_candidates", C.c_int32), ("tpt_max_gamma", C.c_int32),
-                ("tau_conf", C.c_double)]
+                ("tau_conf", C.c_double), ("sampling", KsSampling)]
 
 
 class KsSpecStats(C.Structure):
@@ -74,6 +78,10 @@ _SIGS = {
     "ks_draft": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p]),
     "ks_draft_dynamic": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.c_float, C.c_void_p, C.c_void_p,
                                    C.c_void_p]),
+    "ks_draft_sample": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.POINTER(KsSampling), C.c_uint64,
+                                  C.c_void_p]),
+    "ks_verify_sample": (C.c_int, [C.c_void_p, C.c_int32, C.POINTER(KsSampling), C.c_uint64, C.c_void_p,
+                                   C.c_void_p, C.c_void_p]),
     "ks_verify": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.POINTER(C.c_int32), C.c_void_p,
                             C.POINTER(C.c_int32)]),
     "ks_decode_greedy": (C.c_int, [C.c_void_p, C.c_int32, C.c_void_p]),
@@ -226,6 +234,41 @@ def ks_draft_dynamic(h: int, mask, gamma: int, tau_conf: float, want_outputs: bo
     check(load().ks_draft_dynamic(h, m.ctypes.data, gamma, float(tau_conf), C.byref(n), conf.ctypes.data,
                                   toks.ctypes.data), "ks_draft_dynamic")
     return n.value, conf[: n.value], toks[: n.value]
+
+
+def sampling(temperature: float = 0.7, top_k: int = 50, top_p: float = 0.95, seed: int = 0) -> KsSampling:
+    return KsSampling(float(temperature), int(top_k), float(top_p), int(seed))
+
+
+def ks_draft_sample(h: int, mask, gamma: int, samp: KsSampling, step: int, want_tokens: bool = True):
+    m = np.ascontiguousarray(mask, dtype=np.uint8)
+    out = np.zeros(gamma, np.int32) if want_tokens else None
+    check(load().ks_draft_sample(h, m.ctypes.data, gamma, C.byref(samp), int(step),
+                                 out.ctypes.data if want_tokens else None), "ks_draft_sample")
+    return out
+
+
+def ks_verify_sample(h: int, gamma: int, samp: KsSampling, step: int):
+    """Returns (n_accepted, new tokens array)."""
+    a, n = C.c_int32(), C.c_int32()
+    out = np.zeros(gamma + 1, np.int32)
+    check(load().ks_verify_sample(h, gamma, C.byref(samp), int(step), C.byref(a), out.ctypes.data, C.byref(n)),
+          "ks_verify_sample")
+    return a.value, out[: n.value]
+
+
+def ks_sample_dists(h: int, which: str, start: int, count: int):
+    """Sampling distributions on the device: which = "draft" (q of positions
+    start..) or "target" (p of the last verify rows start..); a list of
+    (ids, probs) per row."""
+    raw = np.zeros((count, 1 + 2 * 64), np.int32)
+    check(load().ks_debug_read(h, 5 if which == "draft" else 6, 0, start, count, raw.ctypes.data, raw.nbytes),
+          "ks_debug_read")
+    out = []
+    for r in range(count):
+        n = int(raw[r, 0])
+        out.append((raw[r, 1:1 + n].astype(np.int64), raw[r, 65:65 + n].view(np.float32).astype(np.float32)))
+    return out
 
 
 def ks_verify(h: int, draft_tokens, gamma: int):

@@ -38,6 +38,13 @@ class Model:
     def draft(self, mask, gamma: int):
         return ks.ks_draft(self.h, mask, gamma)
 
+    def draft_sample(self, mask, gamma: int, samp, step: int):
+        """Sampled drafts (Sec. 2.1, sampling); the draft distributions stay on the device."""
+        return ks.ks_draft_sample(self.h, mask, gamma, samp, step)
+
+    def verify_sample(self, gamma: int, samp, step: int):
+        return ks.ks_verify_sample(self.h, gamma, samp, step)
+
     def draft_dynamic(self, mask, gamma: int, tau_conf: float):
         """Drafts with the dynamic exit (Sec. 3.5): (n_drafted, confidences, tokens)."""
         return ks.ks_draft_dynamic(self.h, mask, gamma, tau_conf)
@@ -52,11 +59,11 @@ class Model:
         return ks.ks_model_position(self.h)
 
     def generate(self, n_tokens: int, gamma: int, mask=None, latency=None, budget_frac: float = 0.5,
-                 resolve_every: int = 64, max_steps: int = 0, tpt=None, tau_conf: float = 0.0):
+                 resolve_every: int = 64, max_steps: int = 0, tpt=None, tau_conf: float = 0.0, sampling=None):
         """Speculative decoding: a fixed mask (policy 0), the knapsack policy
         (policy 1, latency given) or the TPT stage (policy 2, latency and
         tpt = (n_candidates, max_gamma) given); tau_conf > 0 adds the dynamic
-        drafting exit."""
+        drafting exit; sampling (a KsSampling) selects sampling mode."""
         n = self.shape.n_sublayers
         keep = []
         if latency is None:
@@ -74,6 +81,8 @@ class Model:
             else:
                 p = ks.KsSpecParams(gamma, 2, None, lat, 0.0, int(resolve_every), max_steps,
                                     int(tpt[0]), int(tpt[1]), float(tau_conf))
+        if sampling is not None:
+            p.sampling = sampling
         return ks.ks_generate_speculative(self.h, p, n_tokens)
 
     def select_tpt(self, latency, n_candidates: int, max_gamma: int):
