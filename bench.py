@@ -361,6 +361,15 @@ def gpu_arm(args):
                       "alpha": float(sst.accepted) / max(1, sst.drafted),
                       "drafts_per_step": float(sst.drafted) / max(1, sst.steps),
                       "tokens_per_step": n_tok / max(1, sst.steps)})
+        # sampling mode (Sec. 2.1; nucleus sampling with T 0.7, top-k 50, top-p 0.95 as in Sec. 4)
+        p = ks.KsSpecParams(gamma, 1, None, lat, float(args.budget_frac), int(args.resolve_every), 0, 0, 0, 0.0,
+                            ks.sampling(0.7, 50, 0.95, 12345))
+        (o, sst, _a), t = timed(lambda: ks.ks_generate_speculative(h, p, args.e2e_tokens))
+        n_tok = int(sst.steps + sst.accepted)
+        sweep.append({"policy": f"knapsack, gamma {gamma}, budget {args.budget_frac}, sampling T 0.7 top-k 50 top-p 0.95",
+                      "tokens_per_s": n_tok / t, "vs_greedy": (n_tok / t) / ((args.e2e_tokens - 1) / t_ar),
+                      "alpha": float(sst.accepted) / max(1, sst.drafted),
+                      "tokens_per_step": n_tok / max(1, sst.steps)})
 
     ms_max, tok_all = reduce_over_ranks(ms, tokens, dist, "cuda")
 
