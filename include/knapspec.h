@@ -311,6 +311,33 @@ ks_status ks_select_tpt(ks_model* m, const ks_latency* lat, int32_t n_candidates
                         uint8_t* mask_out, int32_t* gamma_out, double* tpt_out, double* alphas_out,
                         uint8_t* candidates_out);
 
+/* NEXT row: the hidden-state dynamic program of Alg. 1 (Sec. 3.4) and the TPT
+ * selection over its candidates (Sec. 3.5, Alg. 2).  On the r most recent
+ * history rows (the last r committed positions, r <= max_rows), g[i, j] is the
+ * best hidden state after sublayer i with skipped weight j (integer weights of
+ * Sec. 3.4 from lat at the committed length): the execute candidate
+ * f^(i)(g[i-1, j]) wins over the skip candidate g[i-1, j - w_i] when its
+ * matrix cosine to the target's X^(i) is at least as high; states with cosine
+ * below tau or j > K / 2 are dropped (Sec. 3.4, pruning; the paper uses tau
+ * 0.5); g[i, 0] = X^(i).  Inside f^(i) a history row attends to the target's
+ * K/V for earlier positions and to the state's own K/V (the target's cache is
+ * restored afterwards).  Each surviving terminal state gives a layer set (by
+ * its recorded choices) and an acceptance estimate (Eq. 4: the fraction of
+ * rows whose LM-head argmax equals the target's); the Eq. 3 grid over the
+ * candidates (executed weight ascending) and gamma = 1..max_gamma picks
+ * (S*, gamma*).
+ * scratch: device, 256-byte aligned, >= ks_dp_scratch_bytes(m, max_states,
+ * max_rows) bytes; max_states (1..128) must cover K / 2 + 1.
+ * Outputs (host): mask_out[2L], *gamma_out, *tpt_out; optional: *n_candidates,
+ * js_out[] (the candidates' skipped weights), alphas_out[], candidates_out
+ * [n][2L] (room for max_states each).  Uses the model's pass buffers; the
+ * decoding state is unchanged.  Waits for the stream (twice). */
+size_t ks_dp_scratch_bytes(const ks_model* m, int32_t max_states, int32_t max_rows);
+ks_status ks_select_dp(ks_model* m, const ks_latency* lat, float tau, int32_t max_gamma, int32_t max_states,
+                       int32_t max_rows, void* scratch, size_t scratch_bytes, uint8_t* mask_out, int32_t* gamma_out,
+                       double* tpt_out, int32_t* n_candidates, int32_t* js_out, double* alphas_out,
+                       uint8_t* candidates_out);
+
 /* ------------------------------------------------- full speculative loop */
 
 typedef struct {

@@ -52,11 +52,12 @@ def _state_kv(session, layer: int):
     return session.k[layer].copy(), session.v[layer].copy()
 
 
-def run_dp(session, hist: np.ndarray, weights, tau: float = 0.5):
+def run_dp(session, hist: np.ndarray, weights, tau: float = 0.5, margins: list | None = None):
     """Alg. 1 over the history rows.  hist: [2L+1, r, d] = X^(0..2L) of the
     last r committed positions; weights: integer w_i of sublayers 1..2L.
     Returns (states, sigma, choices): states[j] = g[2L, j] for the valid
-    terminal j, sigma[j] its cosine to X^(2L), choices[i-1][j] in {"e", "s"}."""
+    terminal j, sigma[j] its cosine to X^(2L), choices[i-1][j] in {"e", "s"}.
+    ``margins``, if given, collects how far each decision was from flipping."""
     hist = np.asarray(hist, np.float64)
     n_sub = hist.shape[0] - 1
     r = hist.shape[1]
@@ -84,6 +85,10 @@ def run_dp(session, hist: np.ndarray, weights, tau: float = 0.5):
                 continue
             se = S.matrix_cos(ce, X) if ce is not None else -np.inf
             ss = S.matrix_cos(cs, X) if cs is not None else -np.inf
+            if margins is not None:      # distance of every decision from its threshold (for tests)
+                if ce is not None and cs is not None:
+                    margins.append(abs(se - ss))
+                margins.append(abs(max(se, ss) - tau))
             if se >= ss:
                 st, s, c = ce, se, "e"
             else:

@@ -13,7 +13,7 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libknapspec.so")
-SOURCES = ["chain.cu", "gemv.cu", "attn.cu", "select.cu", "sample.cu", "model.cu"]
+SOURCES = ["chain.cu", "gemv.cu", "attn.cu", "select.cu", "sample.cu", "dp.cu", "model.cu"]
 HEADERS = ["common.cuh", "internal.h", "tma.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2"]

@@ -177,4 +177,17 @@ struct AcceptSampleArgs {
 cudaError_t launch_filter(const FilterArgs& a, int rows, cudaStream_t s);
 cudaError_t launch_spec_accept(const AcceptSampleArgs& a, cudaStream_t s);
 
+// ------------------------------------------------ hidden-state DP (dp.cu)
+constexpr int kDpMaxStates = 128;   // skipped weights 0 .. 127 (the TPT grid kernel's candidate limit)
+cudaError_t launch_dp_cos(const float* A, long long stride, int n, const float* B, const int32_t* hidx, int r, int d,
+                          float* sig, cudaStream_t s);
+cudaError_t launch_dp_select(int J, int w, float tau, const int* valid_prev, const float* sig_e, const float* sig_s,
+                             int* valid_cur, float* sig_cur, uint8_t* choice, int* src, cudaStream_t s);
+cudaError_t launch_dp_gather(int J, const int* src, const int* valid_cur, const float* E, const float* G_prev,
+                             long long stride, const float* X, const int32_t* hidx, int r, int d, float* G_cur,
+                             cudaStream_t s);
+cudaError_t launch_dp_backtrack(const int* js, int n_cand, int n_items, int J, const uint8_t* choices, const int* w,
+                                uint8_t* masks, cudaStream_t s);
+cudaError_t launch_dp_candidates(int J, const int* valid, int* js, int* n_cand, cudaStream_t s);
+
 }  // namespace ks

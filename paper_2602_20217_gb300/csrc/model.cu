@@ -64,6 +64,27 @@ __global__ void __launch_bounds__(256) embed_kernel(const WT* embed, const int32
     if ((lane & 15) == 0 && k < d) ss[(k / kSsGroup) * 16 + r] = s;
 }
 
+// The pass input taken from rows already in x (the hidden-state DP's states):
+// the 16-feature sums of squares and, for bf16 models, x * gain in bf16, as
+// the embedding kernel leaves them.
+template <typename WT>
+__global__ void __launch_bounds__(256) rows_prep_kernel(const float* x, int d, float* ss, __nv_bfloat16* xg,
+                                                        const WT* gain, const int* stop) {
+    if (stop && *stop) return;
+    const int r = blockIdx.x;
+    const int k = blockIdx.y * 256 + threadIdx.x;
+    float v = 0.f;
+    if (k < d) {
+        v = x[(size_t)r * d + k];
+        if (xg) xg[(size_t)r * d + k] = __float2bfloat16_rn(v * to_float(gain[k]));
+    }
+    float s = v * v;
+#pragma unroll
+    for (int o = 8; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    const int lane = threadIdx.x & 31;
+    if ((lane & 15) == 0 && k < d) ss[(k / kSsGroup) * 16 + r] = s;
+}
+
 // Greedy acceptance (Sec. 2.1): drafts = rows[1..gamma], z = target argmax of
 // rows[0..gamma].  a = longest prefix with drafts[i] == z[i]; the new tokens
 // are drafts[0..a-1] followed by z[a], which becomes the pending rows[0].
@@ -448,6 +469,15 @@ static ks_status forward(ks_model* m, const int32_t* tok, int R, int p0, const u
         g.stop = stop;
     };
     KS_TRY(launch(m, K_EMBED, [&]() -> cudaError_t {
+        if (!tok) {   // input rows already in x
+            if (bf)
+                rows_prep_kernel<__nv_bfloat16><<<dim3(R, (d + 255) / 256), 256, 0, s>>>(
+                    m->x, d, m->ss, m->xg, reinterpret_cast<const __nv_bfloat16*>(next_gain(0)), stop);
+            else
+                rows_prep_kernel<float><<<dim3(R, (d + 255) / 256), 256, 0, s>>>(m->x, d, m->ss, nullptr,
+                                                                                  nullptr, stop);
+            return cudaGetLastError();
+        }
         if (bf)
             embed_kernel<__nv_bfloat16><<<dim3(R, (d + 255) / 256), 256, 0, s>>>(
                 reinterpret_cast<const __nv_bfloat16*>(m->embed), tok, d, c.vocab, m->x, cap_ptr(0), m->ss, m->xg,
@@ -797,7 +827,8 @@ ks_status ks_model_create(const ks_config* cfg, const ks_weights* w, void* works
         delete m;
         return st;
     };
-    m->h_buf_ints = (size_t)cfg->max_seq + 4 * (size_t)R + 64 + lay.hist_slots * (size_t)R + 2 * (size_t)L + 64;
+    m->h_buf_ints = (size_t)cfg->max_seq + 4 * (size_t)R + 64 + lay.hist_slots * (size_t)R + 2 * (size_t)L + 64 +
+                    4 * (size_t)kDpMaxStates + 4 * (size_t)L + 64;   // + the DP stage's staging
     cudaError_t e = cudaHostAlloc(reinterpret_cast<void**>(&m->h_buf), m->h_buf_ints * sizeof(int32_t),
                                   cudaHostAllocDefault);
     if (e != cudaSuccess) {
@@ -1414,6 +1445,257 @@ ks_status ks_select_tpt(ks_model* m, const ks_latency* lat, int32_t n_candidates
     *tpt_out = out[0];
     if (alphas_out)
         for (int j = 0; j < n_candidates; ++j) alphas_out[j] = out[1 + j];
+    return KS_OK;
+}
+
+// ----------------------------------------------- hidden-state DP (Alg. 1)
+// Scratch of ks_select_dp, in this order (256-byte aligned pieces):
+//   G0, G1, E: [S][rows][d] fp32 (states of the previous / current sublayer,
+//   execute candidates); sig_e, sig_s, sig: [S] fp32; valid0, valid1, src,
+//   js: [S] int; n_cand: int; w: [2L] int; choices: [2L][S] u8;
+//   kv: K and V of one layer at the history positions, [2][hk][rows][hd] in
+//   the model dtype; masks: [S][2L] u8; pred: [S + 1][rows] int;
+//   tpt: info[2] int, out[1 + S] double, mask_out[2L] u8.
+struct DpScratch {
+    float *G0, *G1, *E, *sig_e, *sig_s, *sig;
+    int *valid0, *valid1, *src, *js, *n_cand, *w, *pred, *info;
+    uint8_t *choices, *masks, *mask_out;
+    void* kv;
+    double* out;
+    size_t bytes;
+};
+
+static DpScratch dp_layout(const ks_model* m, int S, int rows, char* base) {
+    const ks_config& c = m->cfg;
+    const int nsub = 2 * c.n_layers, d = c.d_model;
+    size_t off = 0;
+    auto take = [&](size_t n) {
+        const size_t o = off;
+        off += align_up(n, 256);
+        return base ? base + o : nullptr;
+    };
+    DpScratch D{};
+    const size_t st = sizeof(float) * (size_t)S * rows * d;
+    D.G0 = reinterpret_cast<float*>(take(st));
+    D.G1 = reinterpret_cast<float*>(take(st));
+    D.E = reinterpret_cast<float*>(take(st));
+    D.sig_e = reinterpret_cast<float*>(take(sizeof(float) * S));
+    D.sig_s = reinterpret_cast<float*>(take(sizeof(float) * S));
+    D.sig = reinterpret_cast<float*>(take(sizeof(float) * S));
+    D.valid0 = reinterpret_cast<int*>(take(sizeof(int) * S));
+    D.valid1 = reinterpret_cast<int*>(take(sizeof(int) * S));
+    D.src = reinterpret_cast<int*>(take(sizeof(int) * S));
+    D.js = reinterpret_cast<int*>(take(sizeof(int) * S));
+    D.n_cand = reinterpret_cast<int*>(take(sizeof(int)));
+    D.w = reinterpret_cast<int*>(take(sizeof(int) * nsub));
+    D.choices = reinterpret_cast<uint8_t*>(take((size_t)nsub * S));
+    D.kv = take(2 * (size_t)c.n_kv_heads * rows * c.head_dim * m->es);
+    D.masks = reinterpret_cast<uint8_t*>(take((size_t)S * nsub));
+    D.pred = reinterpret_cast<int*>(take(sizeof(int) * (size_t)(S + 1) * rows));
+    D.info = reinterpret_cast<int*>(take(sizeof(int) * 2));
+    D.out = reinterpret_cast<double*>(take(sizeof(double) * (1 + (size_t)S)));
+    D.mask_out = reinterpret_cast<uint8_t*>(take((size_t)nsub));
+    D.bytes = off;
+    return D;
+}
+
+size_t ks_dp_scratch_bytes(const ks_model* m, int32_t max_states, int32_t max_rows) {
+    if (!m || max_states < 1 || max_states > kDpMaxStates || max_rows < 1) return 0;
+    return dp_layout(m, max_states, max_rows, nullptr).bytes;
+}
+
+// Integer weights of Sec. 3.4 (the knapsack kernel's rule): Delta = min(t_Attn(n),
+// t_MLP), w = round(t / Delta) half away from zero, at least 1; units as given.
+static void dp_weights(const ks_latency& lat, int64_t n, int nsub, std::vector<int>& w) {
+    w.assign(nsub, 1);
+    if (lat.kind == 1) {
+        for (int i = 0; i < nsub; ++i) w[i] = lat.units[i];
+        return;
+    }
+    volatile double prod = lat.c2 * (double)n;   // two roundings, as the device evaluates c2 n + c3
+    const double ta = prod + lat.c3, tm = lat.c1;
+    const double delta = std::min(ta, tm);
+    const int wa = std::max(1, (int)std::llround(ta / delta)), wm = std::max(1, (int)std::llround(tm / delta));
+    for (int i = 0; i < nsub; ++i) w[i] = (i % 2 == 0) ? wa : wm;
+}
+
+ks_status ks_select_dp(ks_model* m, const ks_latency* lat, float tau, int32_t max_gamma, int32_t max_states,
+                       int32_t max_rows, void* scratch, size_t scratch_bytes, uint8_t* mask_out, int32_t* gamma_out,
+                       double* tpt_out, int32_t* n_candidates, int32_t* js_out, double* alphas_out,
+                       uint8_t* candidates_out) {
+    if (!m || !lat || !scratch || !mask_out || !gamma_out || !tpt_out) {
+        set_error("ks_select_dp: null argument");
+        return KS_ERR_INVALID_ARG;
+    }
+    const ks_config& c = m->cfg;
+    const int nsub = m->nsub, d = c.d_model, L = c.n_layers;
+    if (max_gamma < 1 || max_gamma >= c.max_rows || max_states < 1 || max_states > kDpMaxStates || max_rows < 1 ||
+        !std::isfinite(tau) || !latency_ok(*lat, nsub)) {
+        set_error("ks_select_dp: bad argument");
+        return KS_ERR_INVALID_ARG;
+    }
+    if (!m->have_seq) {
+        set_error("ks_select_dp: no sequence (call ks_prefill first)");
+        return KS_ERR_STATE;
+    }
+    DpScratch D = dp_layout(m, max_states, max_rows, reinterpret_cast<char*>(scratch));
+    if (scratch_bytes < D.bytes || (reinterpret_cast<uintptr_t>(scratch) & 255)) {
+        set_error("ks_select_dp: scratch smaller than ks_dp_scratch_bytes or not 256-byte aligned");
+        return KS_ERR_WORKSPACE;
+    }
+    std::vector<int> w;
+    dp_weights(*lat, m->p, nsub, w);
+    int K = 0;
+    for (int x : w) K += x;
+    const int S = K / 2 + 1;   // skipped weights 0 .. K / 2
+    if (S > max_states) {
+        set_error("ks_select_dp: %d states (K = %d) exceed max_states %d", S, K, max_states);
+        return KS_ERR_CAPACITY;
+    }
+    // history rows: the last r committed positions, oldest first
+    int32_t* hidx = m->h_buf + c.max_seq + 4 * c.max_rows + 16;
+    int r = history_rows(m, hidx);
+    if (r < 1) {
+        set_error("ks_select_dp: empty history");
+        return KS_ERR_STATE;
+    }
+    if (r > max_rows) {   // keep the most recent max_rows rows
+        std::memmove(hidx, hidx + (r - max_rows), sizeof(int32_t) * max_rows);
+        r = max_rows;
+    }
+    const int p0 = m->p - r;
+    cudaStream_t s = m->stream;
+    KS_CUDA(cudaMemcpyAsync(m->hist_idx, hidx, sizeof(int32_t) * r, cudaMemcpyHostToDevice, s), "dp upload");
+    int32_t* hw = m->h_buf + c.max_seq + 4 * c.max_rows + 16 + m->lay.hist_slots * c.max_rows + (nsub + 3) / 4 + 4;
+    std::memcpy(hw, w.data(), sizeof(int) * nsub);
+    KS_CUDA(cudaMemcpyAsync(D.w, hw, sizeof(int) * nsub, cudaMemcpyHostToDevice, s), "dp upload");
+    m->h2d += sizeof(int32_t) * (r + nsub);
+    const long long stride = (long long)r * d;
+    float *Gp = D.G0, *Gc = D.G1;
+    int *vp = D.valid0, *vc = D.valid1;
+    // g[0, 0] = X^(0); every other state starts invalid
+    {
+        std::vector<int> ones(S, 1);
+        ones[0] = 0;
+        int32_t* hv = hw + nsub;
+        std::memcpy(hv, ones.data(), sizeof(int) * S);
+        KS_CUDA(cudaMemcpyAsync(vp, hv, sizeof(int) * S, cudaMemcpyHostToDevice, s), "dp init");
+        ones[0] = -1;
+        std::memcpy(hv + S, ones.data(), sizeof(int) * S);
+        KS_CUDA(cudaMemcpyAsync(D.src, hv + S, sizeof(int) * S, cudaMemcpyHostToDevice, s), "dp init");
+        KS_TRY(launch(m, K_ACCEPT, [&] {
+            return launch_dp_gather(S, D.src, vp, D.E, Gp, stride, hist_plane(m, 0), m->hist_idx, r, d, Gp, s);
+        }, "dp init"));
+    }
+    const size_t kv_row = (size_t)c.head_dim * m->es;
+    const size_t kv_plane = (size_t)c.n_kv_heads * r * kv_row;
+    std::vector<uint8_t> one(nsub, 0);
+    for (int i = 1; i <= nsub; ++i) {
+        const bool attn = (i % 2) == 1;
+        const int l = (i - 1) / 2;
+        std::fill(one.begin(), one.end(), 0);
+        one[i - 1] = 1;
+        char* kc = reinterpret_cast<char*>(kcache(m, l));
+        char* vcach = reinterpret_cast<char*>(vcache(m, l));
+        char* kvs = reinterpret_cast<char*>(D.kv);
+        const size_t seq_pitch = (size_t)c.max_seq * kv_row;
+        if (attn) {   // the target's K/V at the history positions, restored after every state
+            KS_CUDA(cudaMemcpy2DAsync(kvs, r * kv_row, kc + (size_t)p0 * kv_row, seq_pitch, r * kv_row, c.n_kv_heads,
+                                      cudaMemcpyDeviceToDevice, s), "dp kv save");
+            KS_CUDA(cudaMemcpy2DAsync(kvs + kv_plane, r * kv_row, vcach + (size_t)p0 * kv_row, seq_pitch, r * kv_row,
+                                      c.n_kv_heads, cudaMemcpyDeviceToDevice, s), "dp kv save");
+        }
+        for (int j = 1; j < S; ++j) {
+            for (int c0 = 0; c0 < r; c0 += c.max_rows) {
+                const int R = std::min(c.max_rows, r - c0);
+                KS_CUDA(cudaMemcpyAsync(m->x, Gp + (size_t)j * stride + (size_t)c0 * d, sizeof(float) * R * d,
+                                        cudaMemcpyDeviceToDevice, s), "dp state in");
+                KS_TRY(forward(m, nullptr, R, p0 + c0, one.data(), -1, nullptr, vp + j));
+                KS_CUDA(cudaMemcpyAsync(D.E + (size_t)j * stride + (size_t)c0 * d, m->x, sizeof(float) * R * d,
+                                        cudaMemcpyDeviceToDevice, s), "dp state out");
+            }
+            if (attn) {
+                KS_CUDA(cudaMemcpy2DAsync(kc + (size_t)p0 * kv_row, seq_pitch, kvs, r * kv_row, r * kv_row,
+                                          c.n_kv_heads, cudaMemcpyDeviceToDevice, s), "dp kv restore");
+                KS_CUDA(cudaMemcpy2DAsync(vcach + (size_t)p0 * kv_row, seq_pitch, kvs + kv_plane, r * kv_row,
+                                          r * kv_row, c.n_kv_heads, cudaMemcpyDeviceToDevice, s), "dp kv restore");
+            }
+        }
+        const float* X = hist_plane(m, i);
+        KS_TRY(launch(m, K_ACCEPT, [&] { return launch_dp_cos(D.E, stride, S, X, m->hist_idx, r, d, D.sig_e, s); },
+                      "dp cosines"));
+        KS_TRY(launch(m, K_ACCEPT, [&] { return launch_dp_cos(Gp, stride, S, X, m->hist_idx, r, d, D.sig_s, s); },
+                      "dp cosines"));
+        KS_TRY(launch(m, K_ACCEPT, [&] {
+            return launch_dp_select(S, w[i - 1], tau, vp, D.sig_e, D.sig_s, vc, D.sig, D.choices + (size_t)(i - 1) * S,
+                                    D.src, s);
+        }, "dp select"));
+        KS_TRY(launch(m, K_ACCEPT, [&] {
+            return launch_dp_gather(S, D.src, vc, D.E, Gp, stride, X, m->hist_idx, r, d, Gc, s);
+        }, "dp gather"));
+        std::swap(Gp, Gc);
+        std::swap(vp, vc);
+    }
+    // terminal candidates, executed weight ascending
+    KS_TRY(launch(m, K_ACCEPT, [&] { return launch_dp_candidates(S, vp, D.js, D.n_cand, s); }, "dp candidates"));
+    int32_t* hc = hw + nsub;
+    KS_CUDA(cudaMemcpyAsync(hc, D.n_cand, sizeof(int), cudaMemcpyDeviceToHost, s), "dp candidates");
+    KS_CUDA(cudaMemcpyAsync(hc + 1, D.js, sizeof(int) * S, cudaMemcpyDeviceToHost, s), "dp candidates");
+    m->d2h += sizeof(int) * (1 + S);
+    KS_TRY(sync(m, "ks_select_dp"));
+    const int n_cand = hc[0];
+    std::vector<int> js(hc + 1, hc + 1 + n_cand);
+    if (n_cand < 1) {
+        set_error("ks_select_dp: no state survived the pruning (tau %g)", (double)tau);
+        return KS_ERR_STATE;
+    }
+    KS_TRY(launch(m, K_ACCEPT, [&] {
+        return launch_dp_backtrack(D.js, n_cand, nsub, S, D.choices, D.w, D.masks, s);
+    }, "dp backtrack"));
+    // Eq. 4 inputs: the LM head's argmax of every terminal state's rows and of X^(2L)
+    for (int cnd = 0; cnd <= n_cand; ++cnd) {
+        for (int c0 = 0; c0 < r; c0 += c.max_rows) {
+            const int R = std::min(c.max_rows, r - c0);
+            if (cnd < n_cand) {
+                KS_CUDA(cudaMemcpyAsync(m->x, Gp + (size_t)js[cnd] * stride + (size_t)c0 * d, sizeof(float) * R * d,
+                                        cudaMemcpyDeviceToDevice, s), "dp prediction rows");
+            } else {   // the target's rows X^(2L) (gathered like state 0 of sublayer 2L)
+                KS_CUDA(cudaMemcpyAsync(m->x, Gp + (size_t)c0 * d, sizeof(float) * R * d, cudaMemcpyDeviceToDevice,
+                                        s), "dp prediction rows");
+            }
+            KS_TRY(launch(m, K_EMBED, [&]() -> cudaError_t {
+                if (m->dtype == KS_DTYPE_BF16)
+                    rows_prep_kernel<__nv_bfloat16><<<dim3(R, (d + 255) / 256), 256, 0, s>>>(
+                        m->x, d, m->ss, m->xg, reinterpret_cast<const __nv_bfloat16*>(m->final_norm), nullptr);
+                else
+                    rows_prep_kernel<float><<<dim3(R, (d + 255) / 256), 256, 0, s>>>(m->x, d, m->ss, nullptr, nullptr,
+                                                                                      nullptr);
+                return cudaGetLastError();
+            }, "dp prediction prep"));
+            KS_TRY(lm_head_rows(m, R, D.pred + (size_t)cnd * r + c0));
+        }
+    }
+    KS_TRY(launch(m, K_ACCEPT, [&] {
+        return launch_tpt(lat, m->p, nsub, L, n_cand, r, max_gamma, D.masks, D.pred, D.mask_out, D.info, D.out, s);
+    }, "dp tpt grid"));
+    std::vector<double> outv(1 + n_cand);
+    int32_t info[2] = {0, 0};
+    KS_CUDA(cudaMemcpyAsync(mask_out, D.mask_out, nsub, cudaMemcpyDeviceToHost, s), "dp download");
+    KS_CUDA(cudaMemcpyAsync(info, D.info, sizeof(info), cudaMemcpyDeviceToHost, s), "dp download");
+    KS_CUDA(cudaMemcpyAsync(outv.data(), D.out, sizeof(double) * outv.size(), cudaMemcpyDeviceToHost, s),
+            "dp download");
+    if (candidates_out)
+        KS_CUDA(cudaMemcpyAsync(candidates_out, D.masks, (size_t)n_cand * nsub, cudaMemcpyDeviceToHost, s),
+                "dp download");
+    m->d2h += nsub + sizeof(info) + sizeof(double) * outv.size() + (candidates_out ? (size_t)n_cand * nsub : 0);
+    KS_TRY(sync(m, "ks_select_dp"));
+    *gamma_out = info[1];
+    *tpt_out = outv[0];
+    if (n_candidates) *n_candidates = n_cand;
+    if (js_out)
+        for (int k = 0; k < n_cand; ++k) js_out[k] = js[k];
+    if (alphas_out)
+        for (int k = 0; k < n_cand; ++k) alphas_out[k] = outv[1 + k];
     return KS_OK;
 }
 

@@ -71,7 +71,7 @@ cudaError_t launch_cosine(const void* X, const void* Y, int dtype, int64_t n_pai
 
 // ----------------------------------------------------------------- knapsack
 constexpr int kMaxItems = 256;
-constexpr int kMaxTpt = KS_TPT_MAX_CANDIDATES;
+constexpr int kMaxTpt = 128;   // ks_select_tpt passes at most KS_TPT_MAX_CANDIDATES; the DP stage more
 constexpr int kKnapThreads = 512;
 
 struct KnapArgs {

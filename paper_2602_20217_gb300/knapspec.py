@@ -78,6 +78,10 @@ _SIGS = {
     "ks_draft": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p]),
     "ks_draft_dynamic": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.c_float, C.c_void_p, C.c_void_p,
                                    C.c_void_p]),
+    "ks_dp_scratch_bytes": (C.c_size_t, [C.c_void_p, C.c_int32, C.c_int32]),
+    "ks_select_dp": (C.c_int, [C.c_void_p, C.POINTER(KsLatency), C.c_float, C.c_int32, C.c_int32, C.c_int32,
+                               C.c_void_p, C.c_size_t, C.c_void_p, C.POINTER(C.c_int32), C.POINTER(C.c_double),
+                               C.POINTER(C.c_int32), C.c_void_p, C.c_void_p, C.c_void_p]),
     "ks_draft_sample": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.POINTER(KsSampling), C.c_uint64,
                                   C.c_void_p]),
     "ks_verify_sample": (C.c_int, [C.c_void_p, C.c_int32, C.POINTER(KsSampling), C.c_uint64, C.c_void_p,
@@ -269,6 +273,21 @@ def ks_sample_dists(h: int, which: str, start: int, count: int):
         n = int(raw[r, 0])
         out.append((raw[r, 1:1 + n].astype(np.int64), raw[r, 65:65 + n].view(np.float32).astype(np.float32)))
     return out
+
+
+def ks_select_dp(h: int, lat: KsLatency, n_sublayers: int, tau: float, max_gamma: int, max_states: int,
+                 max_rows: int, scratch_ptr: int, scratch_bytes: int):
+    """Alg. 1 + the TPT grid: (mask, gamma, tpt, js, alphas, candidate masks)."""
+    mask = np.zeros(n_sublayers, np.uint8)
+    g, tpt, n = C.c_int32(), C.c_double(), C.c_int32()
+    js = np.zeros(max_states, np.int32)
+    alphas = np.zeros(max_states, np.float64)
+    cands = np.zeros((max_states, n_sublayers), np.uint8)
+    check(load().ks_select_dp(h, C.byref(lat), float(tau), max_gamma, max_states, max_rows, scratch_ptr,
+                              scratch_bytes, mask.ctypes.data, C.byref(g), C.byref(tpt), C.byref(n), js.ctypes.data,
+                              alphas.ctypes.data, cands.ctypes.data), "ks_select_dp")
+    k = n.value
+    return mask, g.value, tpt.value, js[:k].copy(), alphas[:k].copy(), cands[:k].copy()
 
 
 def ks_verify(h: int, draft_tokens, gamma: int):

@@ -85,6 +85,18 @@ class Model:
             p.sampling = sampling
         return ks.ks_generate_speculative(self.h, p, n_tokens)
 
+    def select_dp(self, latency, max_gamma: int, tau: float = 0.5, max_states: int = 128, max_rows: int = 32):
+        """Alg. 1 on the current history and the TPT grid over its candidates:
+        (mask, gamma, tpt, js, alphas, candidate masks)."""
+        import torch
+        lat, _u = latency
+        nb = ks.load().ks_dp_scratch_bytes(self.h, max_states, max_rows)
+        if nb == 0:
+            raise ValueError("bad max_states / max_rows")
+        scratch = torch.empty(nb + 256, dtype=torch.uint8, device=self.workspace.device)
+        ptr = (scratch.data_ptr() + 255) // 256 * 256
+        return ks.ks_select_dp(self.h, lat, self.shape.n_sublayers, tau, max_gamma, max_states, max_rows, ptr, nb)
+
     def select_tpt(self, latency, n_candidates: int, max_gamma: int):
         """The TPT stage on the current history: (mask, gamma, tpt, alphas, candidates)."""
         lat, _u = latency
