@@ -361,6 +361,26 @@ def gpu_arm(args):
                       "alpha": float(sst.accepted) / max(1, sst.drafted),
                       "drafts_per_step": float(sst.drafted) / max(1, sst.steps),
                       "tokens_per_step": n_tok / max(1, sst.steps)})
+        # Alg. 1 (hidden-state DP, tau 0.5) + the Eq. 3 grid on a filled history, then the
+        # e2e job decoded with the (S*, gamma*) it picks
+        rewind()
+        ks.ks_generate_speculative(h, ks.KsSpecParams(gamma, 1, None, lat, float(args.budget_frac),
+                                                      int(args.resolve_every), 6), 1 << 20)
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        dmask, dgamma, dtpt, djs, dalphas, dcands = model.select_dp((lat, _keep), tpt_d, tau=0.5, max_states=128,
+                                                                    max_rows=32)
+        dp_s = time.perf_counter() - t0
+        dm = np.ascontiguousarray(dmask, np.uint8)
+        p = ks.KsSpecParams(int(dgamma), 0, dm.ctypes.data_as(ks.C.POINTER(ks.C.c_uint8)), lat, 0.0, 1, 0)
+        (o, sst, _a), t = timed(lambda: ks.ks_generate_speculative(h, p, args.e2e_tokens))
+        n_tok = int(sst.steps + sst.accepted)
+        sweep.append({"policy": f"hidden-state DP (Alg. 1, tau 0.5) + TPT grid (D {tpt_d}), selected once",
+                      "dp_seconds": dp_s, "dp_candidates": int(len(djs)), "gamma": int(dgamma),
+                      "skipped_attn_mlp": [int(np.sum(dmask[0::2] == 0)), int(np.sum(dmask[1::2] == 0))],
+                      "tokens_per_s": n_tok / t, "vs_greedy": (n_tok / t) / ((args.e2e_tokens - 1) / t_ar),
+                      "alpha": float(sst.accepted) / max(1, sst.drafted),
+                      "tokens_per_step": n_tok / max(1, sst.steps)})
         # sampling mode (Sec. 2.1; nucleus sampling with T 0.7, top-k 50, top-p 0.95 as in Sec. 4)
         p = ks.KsSpecParams(gamma, 1, None, lat, float(args.budget_frac), int(args.resolve_every), 0, 0, 0, 0.0,
                             ks.sampling(0.7, 50, 0.95, 12345))
