@@ -71,7 +71,14 @@ KS_DEV void set_err(int* e, int code) { atomicCAS(e, 0, code); }
 
 struct Phase {
     int kind, layer, N, K, n_items, tpi;
+    int n_sl, sl_len, n_units;   // K-slices per item (residual phases with few items), stages per slice
 };
+
+// The residual projections W_o and W_down have only d / 16 row groups (256 for
+// d = 4096): fewer items than CTAs.  Their items are split into two K-slices
+// (fixed by the shape, never by R, so every row has the same arithmetic);
+// the slice that finishes second adds both partial sums in slice order.
+constexpr int kSliceMaxItems = kChainSliceMaxItems;
 
 KS_DEV Phase decode(const ChainArgs& a, int k) {
     const int code = a.code[k];
@@ -91,6 +98,9 @@ KS_DEV Phase decode(const ChainArgs& a, int k) {
     p.n_items = (p.N + 15) >> 4;
     const int cols = p.kind == CH_GU ? 512 : 1024;   // k columns per stage
     p.tpi = (p.K + cols - 1) / cols;
+    p.n_sl = ((p.kind == CH_O || p.kind == CH_DOWN) && p.n_items <= kSliceMaxItems && p.tpi >= 2) ? 2 : 1;
+    p.sl_len = (p.tpi + p.n_sl - 1) / p.n_sl;
+    p.n_units = p.n_items * p.n_sl;
     return p;
 }
 KS_DEV bool normed_input(int kind) { return kind == CH_QKV || kind == CH_GU || kind == CH_LM; }
@@ -264,9 +274,11 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
     __shared__ __align__(8) uint64_t pub[kMaxStages];
     __shared__ int slot_k[kMaxStages], slot_it[kMaxStages], slot_kt[kMaxStages];
     __shared__ int slot_last[kMaxStages];   // the stage ends this CTA's last item of its phase
+    __shared__ int slot_sl[kMaxStages];     // the item's K-slice
+    __shared__ float ones[kMaxRows];        // the input scale of phases without a norm
     __shared__ float scale[2][kMaxRows];
     __shared__ float red[2][4][2][NT * 4][32];   // [buffer][consumer warp][gate, up][fragment][lane]
-    __shared__ int red_k[2], red_it[2], red_last[2];
+    __shared__ int red_k[2], red_it[2], red_last[2], red_sl[2];
     __shared__ __align__(8) uint64_t red_full[2];   // 4 consumer warps arrive
     __shared__ __align__(8) uint64_t red_free[2];   // the epilogue warp arrives
 
@@ -290,6 +302,7 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
         }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
+    if (tid < kMaxRows) ones[tid] = 1.f;
     __syncthreads();
 
     if (warp == kWarpW) {
@@ -297,10 +310,11 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
         if (lane == 0) {
             bool ok = true;
             int t = 0;
-            auto issue = [&](int k, const Phase& P, int it, int kt, bool last_item) -> bool {
+            auto issue = [&](int k, const Phase& P, int it, int kt, int sl, bool last_item) -> bool {
                 const int slot = t % S;
                 // self-check: every box coordinate below follows from these ranges
-                if (k < 0 || k >= a.n_phases || it < 0 || it >= P.n_items || kt < 0 || kt >= P.tpi) {
+                if (k < 0 || k >= a.n_phases || it < 0 || it >= P.n_items || kt < 0 || kt >= P.tpi || sl < 0 ||
+                    sl >= P.n_sl) {
                     set_err(a.err, kErrCheckW);
                     return false;
                 }
@@ -309,6 +323,7 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
                 slot_it[slot] = it;
                 slot_kt[slot] = kt;
                 slot_last[slot] = last_item;
+                slot_sl[slot] = sl;
                 mbar_expect_tx(&full[slot], kWBytes);
                 __nv_bfloat16* st = ring + (size_t)slot * stage_elems;
                 const CUtensorMap* wm = &a.wmap[k];
@@ -340,17 +355,20 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
             int k = 0;
             Phase P = decode(a, 0);
             int it = atomicAdd(&queue[0], 1);
-            while (ok) {
-                if (it >= P.n_items) {
+            while (ok) {   // `it` counts units: item it / n_sl, K-slice it % n_sl
+                if (it >= P.n_units) {
                     if (++k >= a.n_phases) break;
                     P = decode(a, k);
                     it = atomicAdd(&queue[k], 1);
                     continue;
                 }
                 const int next = atomicAdd(&queue[k], 1);  // claimed ahead: its latency hides behind the stream
-                // (the ticket is first needed at the item's last stage, so its
-                // round trip overlaps the item's other stages)
-                for (int kt = 0; kt < P.tpi && ok; ++kt) ok = issue(k, P, it, kt, kt == P.tpi - 1 && next >= P.n_items);
+                // (the ticket is first needed at the unit's last stage, so its
+                // round trip overlaps the unit's other stages)
+                const int item = it / P.n_sl, sl = it - item * P.n_sl;
+                const int kt0 = sl * P.sl_len, kt1 = min(P.tpi, kt0 + P.sl_len);
+                for (int kt = kt0; kt < kt1 && ok; ++kt)
+                    ok = issue(k, P, item, kt, sl, kt == kt1 - 1 && next >= P.n_units);
                 it = next;
             }
             if (ok) {  // sentinel stage: no more work
@@ -465,7 +483,7 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
                 break;
             }
             const int k = slot_k[slot];
-            const int it = slot_it[slot], kt = slot_kt[slot];
+            const int it = slot_it[slot], kt = slot_kt[slot], sl = slot_sl[slot];
             const bool last_item = slot_last[slot] != 0;
             const int b = n_items & 1;
             if (k < 0) {
@@ -483,12 +501,13 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
                 break;
             }
             const Phase P = decode(a, k);
-            if (kt >= P.tpi || it >= P.n_items) {
+            if (kt >= P.tpi || it >= P.n_items || sl < 0 || sl >= P.n_sl) {
                 if (lane == 0) set_err(a.err, kErrCheckC);
                 failed = true;
                 break;
             }
-            if (kt == 0) {
+            const int kt0 = sl * P.sl_len, kt1 = min(P.tpi, kt0 + P.sl_len);
+            if (kt == kt0) {
 #pragma unroll
                 for (int c = 0; c < kChains; ++c)
 #pragma unroll
@@ -501,7 +520,7 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
             else mma_stage<NT, false>(st, R, warp, lane, acc, accu);
             __syncwarp();
             if (lane == 0) mbar_arrive(&empty[slot]);   // this warp is done with the stage
-            if (kt != P.tpi - 1) continue;
+            if (kt != kt1 - 1) continue;
 
             // item done: add the chains in chain order and hand this warp's
             // sums to the epilogue warp through partials buffer b (double
@@ -530,6 +549,7 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
                 red_k[b] = k;
                 red_it[b] = it;
                 red_last[b] = last_item;
+                red_sl[b] = sl;
             }
             __syncwarp();
             if (lane == 0) mbar_arrive(&red_full[b]);
@@ -584,11 +604,47 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
                         acc[nt][i] += red[b][w][0][nt * 4 + i][lane];
                         if (P.kind == CH_GU) accu[nt][i] += red[b][w][1][nt * 4 + i][lane];
                     }
+            const int sl = red_sl[b];
             __syncwarp();
             if (lane == 0) mbar_arrive(&red_free[b]);   // partials read: the buffer is free
-            epilogue<NT>(a, P, k, it, acc, accu, scale[k & 1], run_v, run_i);
-            ++items_in_phase;
-            if (k + 1 < a.n_phases) {
+            bool complete = true;
+            if (P.n_sl > 1) {
+                // a K-slice: leave its sums in global memory; the slice that
+                // completes the item adds all of them in slice order
+                const int g = lane >> 2, t4 = lane & 3;
+                float* part = a.slice_part + ((size_t)(k & 1) * kSliceMaxItems + it) * (2 * 256);
+#pragma unroll
+                for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+                        part[sl * 256 + (g + 8 * (i >> 1)) * 16 + nt * 8 + 2 * t4 + (i & 1)] = acc[nt][i];
+                __syncwarp();
+                int last = 0;
+                if (lane == 0) {
+                    __threadfence();
+                    int* tk = a.slice_ticket + (k & 1) * kSliceMaxItems + it;
+                    last = atomicAdd(tk, 1) == P.n_sl - 1;
+                    if (last) *tk = 0;   // every slice has arrived: ready for the next use
+                }
+                complete = __shfl_sync(0xffffffffu, last, 0) != 0;
+                if (complete) {
+                    __threadfence();
+#pragma unroll
+                    for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) {
+                            const int o = (g + 8 * (i >> 1)) * 16 + nt * 8 + 2 * t4 + (i & 1);
+                            float v = __ldcg(&part[o]);
+                            for (int q = 1; q < P.n_sl; ++q) v += __ldcg(&part[q * 256 + o]);
+                            acc[nt][i] = v;
+                        }
+                }
+            }
+            if (complete) {
+                epilogue<NT>(a, P, k, it, acc, accu, normed_input(P.kind) ? scale[k & 1] : ones, run_v, run_i);
+                ++items_in_phase;
+            }
+            if (complete && k + 1 < a.n_phases) {
                 // publish this row group to the next phase's stages that read it
                 fence_proxy_async_global();
                 __syncwarp();

@@ -75,6 +75,7 @@ int gemv_groups(int N, int dtype);              // output groups (argmax candida
 constexpr int kChainMaxPhases = 160;
 enum ChainKind { CH_QKV = 0, CH_O = 1, CH_GU = 2, CH_DOWN = 3, CH_LM = 4 };
 
+constexpr int kChainSliceMaxItems = 640;   // residual phases with at most this many row groups are K-sliced
 struct ChainArgs {
     CUtensorMap wmap[kChainMaxPhases];  // weights of each phase (make_weight_map)
     CUtensorMap amap[4];        // inputs for this R: xg (4-chunk stages), xg (2-chunk), attn_out, act
@@ -96,6 +97,8 @@ struct ChainArgs {
     int* counters;              // chain_counter_ints() zeros; the launch leaves them zero
     int* err;                   // device status word
     const int* stop;            // draft passes: the launch does nothing when *stop != 0 (null: always)
+    float* slice_part;          // K-sliced residual phases: [2][kChainSliceMaxItems][2][16][16] partial sums
+    int* slice_ticket;          // [2][kChainSliceMaxItems] arrivals per item (zero between uses)
     uint16_t code[kChainMaxPhases];
     const __nv_bfloat16* gain[kChainMaxPhases];  // O / down phases: gain of the next RMSNorm
 };

@@ -181,7 +181,7 @@ static size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 struct Layout {
     size_t kv, rope, x, ss, xg, qkv, attn_out, act, attn_part, gemv_part, counters, logits, amax_val,
         amax_idx, tok, hist, hist_snap, hist_idx, sims, mask, obj, wts, select, chain_ctr, best, tpt_masks,
-        tpt_tok, tpt_info, tpt_out, dyn, samp, total;
+        tpt_tok, tpt_info, tpt_out, dyn, samp, slice, total;
     int n_chunks_max;
     size_t gemv_part_floats;
     int counters_n;
@@ -272,6 +272,8 @@ static Layout make_layout(const ks_config* c) {
     L.dyn = take(sizeof(float) * ((size_t)R + kTop1Ctas) + sizeof(int));
     // sampling: q and p distributions, [R][kSampleMaxK] ids and probs plus [R] sizes each
     L.samp = take(2 * ((size_t)R * kSampleMaxK * (sizeof(int) + sizeof(float)) + sizeof(int) * R));
+    // chain kernel K-slices: partial sums [2][640][2][16][16] floats, then tickets [2][640]
+    L.slice = take(sizeof(float) * 2 * kChainSliceMaxItems * 512 + sizeof(int) * 2 * kChainSliceMaxItems);
     L.total = off;
     return L;
 }
@@ -319,6 +321,8 @@ struct ks_model {
     int* top1_ticket;
     int* stop;                // dynamic exit: set once a draft token is below tau_conf
     int* n_drafted;           // dynamic exit: draft passes of the step that ran
+    float* slice_part;        // chain kernel: K-slice partial sums
+    int* slice_ticket;
     bool last_dynamic = false;
     bool last_sampled = false;   // the drafts on the device were sampled (ks_draft_sample)
     int *q_ids, *q_n, *p_ids, *p_n;   // sampling mode: draft / target distributions [16][kSampleMaxK]
@@ -535,6 +539,8 @@ static ks_status forward(ks_model* m, const int32_t* tok, int R, int p0, const u
         ca.capture_plane = (long long)m->lay.hist_slots * c.max_rows * d;
         ca.err = m->err;
         ca.stop = stop;
+        ca.slice_part = m->slice_part;
+        ca.slice_ticket = m->slice_ticket;
         int nph = 0, klass = K_CHAIN;
         double bytes = 0.0;
         auto flush = [&]() -> ks_status {
@@ -778,6 +784,8 @@ ks_status ks_model_create(const ks_config* cfg, const ks_weights* w, void* works
     m->top1_ticket = reinterpret_cast<int*>(m->top1_part + kTop1Ctas);
     m->stop = m->rows + (3 * cfg->max_rows + 5);        // spare words of the token block
     m->n_drafted = m->rows + (3 * cfg->max_rows + 6);
+    m->slice_part = reinterpret_cast<float*>(b + lay.slice);
+    m->slice_ticket = reinterpret_cast<int*>(m->slice_part + (size_t)2 * kChainSliceMaxItems * 512);
     {
         char* sb = b + lay.samp;
         const size_t RK = (size_t)cfg->max_rows * kSampleMaxK;
@@ -860,6 +868,8 @@ ks_status ks_model_create(const ks_config* cfg, const ks_weights* w, void* works
     if (e != cudaSuccess) return fail(e, "counter reset");
     e = cudaMemsetAsync(b + lay.tok, 0, sizeof(int) * ((size_t)3 * R + 8 + cfg->max_seq), m->stream);  // incl. err
     if (e != cudaSuccess) return fail(e, "token reset");
+    e = cudaMemsetAsync(m->slice_ticket, 0, sizeof(int) * 2 * kChainSliceMaxItems, m->stream);
+    if (e != cudaSuccess) return fail(e, "slice reset");
     e = cudaMemsetAsync(b + lay.dyn, 0, sizeof(float) * ((size_t)R + kTop1Ctas) + sizeof(int), m->stream);
     if (e != cudaSuccess) return fail(e, "dynamic-exit reset");
     e = cudaStreamSynchronize(m->stream);
@@ -1291,6 +1301,8 @@ static ks_status lm_head_rows(ks_model* m, int R, int32_t* tokens) {
         ca.capture = nullptr;
         ca.err = m->err;
         ca.stop = nullptr;
+        ca.slice_part = m->slice_part;
+        ca.slice_ticket = m->slice_ticket;
         ca.n_phases = 1;
         ca.code[0] = (uint16_t)(4 * L);
         ca.gain[0] = nullptr;
