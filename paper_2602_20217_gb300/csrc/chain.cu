@@ -75,9 +75,11 @@ struct Phase {
 };
 
 // The residual projections W_o and W_down have only d / 16 row groups (256 for
-// d = 4096): fewer items than CTAs.  Their items are split into two K-slices
-// (fixed by the shape, never by R, so every row has the same arithmetic);
-// the slice that finishes second adds both partial sums in slice order.
+// d = 4096): fewer items than CTAs.  Long items (8 stages or more: W_down, and
+// W_o at hq * hd >= 8192) are split into two K-slices (fixed by the shape,
+// never by R, so every row has the same arithmetic); the slice that finishes
+// second adds both partial sums in slice order.  Short items stay whole: a
+// slice's partial-sum round trip would cost more than it balances.
 constexpr int kSliceMaxItems = kChainSliceMaxItems;
 
 KS_DEV Phase decode(const ChainArgs& a, int k) {
@@ -98,7 +100,7 @@ KS_DEV Phase decode(const ChainArgs& a, int k) {
     p.n_items = (p.N + 15) >> 4;
     const int cols = p.kind == CH_GU ? 512 : 1024;   // k columns per stage
     p.tpi = (p.K + cols - 1) / cols;
-    p.n_sl = ((p.kind == CH_O || p.kind == CH_DOWN) && p.n_items <= kSliceMaxItems && p.tpi >= 2) ? 2 : 1;
+    p.n_sl = ((p.kind == CH_O || p.kind == CH_DOWN) && p.n_items <= kSliceMaxItems && p.tpi >= 8) ? 2 : 1;
     p.sl_len = (p.tpi + p.n_sl - 1) / p.n_sl;
     p.n_units = p.n_items * p.n_sl;
     return p;
