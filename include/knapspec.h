@@ -345,7 +345,8 @@ typedef struct {
                                 the first selection                                         */
     int32_t policy;          /* 0 fixed mask; 1 knapsack re-solved every resolve_every steps;
                                 2 TPT stage (ks_select_tpt) every resolve_every steps, which
-                                also sets gamma                                             */
+                                also sets gamma; 3 the hidden-state DP (ks_select_dp) every
+                                resolve_every steps, which also sets gamma                   */
     const uint8_t* mask;     /* host uint8[2L]: the mask for policy 0                      */
     ks_latency latency;      /* policies 1 and 2                                            */
     double budget_frac;      /* policy 1: budget = floor(budget_frac * sum_i w_i)          */
@@ -358,6 +359,12 @@ typedef struct {
     ks_sampling sampling;    /* temperature > 0: sampling mode (ks_draft_sample /
                                 ks_verify_sample, step = the verify step index from 0);
                                 not combined with tau_conf                                 */
+    void* dp_scratch;        /* policy 3: scratch of ks_select_dp (caller-owned, device)    */
+    uint64_t dp_scratch_bytes;
+    float dp_tau;            /* policy 3: tau of ks_select_dp                               */
+    int32_t dp_max_states;   /* policy 3: max_states / max_rows of ks_select_dp; its
+                                max_gamma is tpt_max_gamma                                 */
+    int32_t dp_max_rows;
 } ks_spec_params;
 
 typedef struct {

@@ -1722,11 +1722,13 @@ ks_status ks_generate_speculative(ks_model* m, const ks_spec_params* prm, int32_
         return KS_ERR_STATE;
     }
     const int nsub = m->nsub;
-    if (prm->gamma < 1 || prm->gamma >= m->cfg.max_rows || prm->policy < 0 || prm->policy > 2 ||
+    if (prm->gamma < 1 || prm->gamma >= m->cfg.max_rows || prm->policy < 0 || prm->policy > 3 ||
         (prm->policy == 0 && !prm->mask) ||
         (prm->policy == 1 && (prm->resolve_every < 1 || !(prm->budget_frac >= 0.0) || prm->budget_frac > 1.0)) ||
         (prm->policy == 2 && (prm->resolve_every < 1 || prm->tpt_candidates < 1 ||
                               prm->tpt_candidates > KS_TPT_MAX_CANDIDATES || prm->tpt_max_gamma < 1 ||
+                              prm->tpt_max_gamma >= m->cfg.max_rows)) ||
+        (prm->policy == 3 && (prm->resolve_every < 1 || !prm->dp_scratch || prm->tpt_max_gamma < 1 ||
                               prm->tpt_max_gamma >= m->cfg.max_rows))) {
         set_error("ks_generate_speculative: bad parameters");
         return KS_ERR_INVALID_ARG;
@@ -1766,6 +1768,16 @@ ks_status ks_generate_speculative(ks_model* m, const ks_spec_params* prm, int32_
             KS_TRY(sync(m, "select"));
             std::memcpy(mask.data(), hm, nsub);
             gamma = hg[1];
+            st.resolves++;
+        }
+        if (prm->policy == 3 && st.steps % prm->resolve_every == 0) {
+            // Alg. 1 + the Eq. 3 grid: the next mask and draft length
+            int32_t gsel = 0;
+            double tsel = 0.0;
+            KS_TRY(ks_select_dp(m, &prm->latency, prm->dp_tau, prm->tpt_max_gamma, prm->dp_max_states,
+                                prm->dp_max_rows, prm->dp_scratch, (size_t)prm->dp_scratch_bytes, mask.data(),
+                                &gsel, &tsel, nullptr, nullptr, nullptr, nullptr));
+            gamma = gsel;
             st.resolves++;
         }
         if (prm->policy == 1 && st.steps % prm->resolve_every == 0) {

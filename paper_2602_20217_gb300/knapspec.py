@@ -52,7 +52,9 @@ class KsSpecParams(C.Structure):
     _fields_ = [("gamma", C.c_int32), ("policy", C.c_int32), ("mask", C.POINTER(C.c_uint8)),
                 ("latency", KsLatency), ("budget_frac", C.c_double), ("resolve_every", C.c_int32),
                 ("max_steps", C.c_int32), ("tpt_candidates", C.c_int32), ("tpt_max_gamma", C.c_int32),
-                ("tau_conf", C.c_double), ("sampling", KsSampling)]
+                ("tau_conf", C.c_double), ("sampling", KsSampling), ("dp_scratch", C.c_void_p),
+                ("dp_scratch_bytes", C.c_uint64), ("dp_tau", C.c_float), ("dp_max_states", C.c_int32),
+                ("dp_max_rows", C.c_int32)]
 
 
 class KsSpecStats(C.Structure):

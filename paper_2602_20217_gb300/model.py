@@ -59,11 +59,13 @@ class Model:
         return ks.ks_model_position(self.h)
 
     def generate(self, n_tokens: int, gamma: int, mask=None, latency=None, budget_frac: float = 0.5,
-                 resolve_every: int = 64, max_steps: int = 0, tpt=None, tau_conf: float = 0.0, sampling=None):
+                 resolve_every: int = 64, max_steps: int = 0, tpt=None, tau_conf: float = 0.0, sampling=None,
+                 dp=None):
         """Speculative decoding: a fixed mask (policy 0), the knapsack policy
         (policy 1, latency given) or the TPT stage (policy 2, latency and
         tpt = (n_candidates, max_gamma) given); tau_conf > 0 adds the dynamic
-        drafting exit; sampling (a KsSampling) selects sampling mode."""
+        drafting exit; sampling (a KsSampling) selects sampling mode; dp = (max_gamma, tau,
+        max_states, max_rows) with a latency selects the hidden-state DP policy."""
         n = self.shape.n_sublayers
         keep = []
         if latency is None:
@@ -83,7 +85,23 @@ class Model:
                                     int(tpt[0]), int(tpt[1]), float(tau_conf))
         if sampling is not None:
             p.sampling = sampling
-        return ks.ks_generate_speculative(self.h, p, n_tokens)
+        scratch = None
+        if dp is not None:
+            # policy 3: the hidden-state DP every resolve_every steps; dp = (max_gamma, tau, max_states, max_rows)
+            import torch
+            D, tau, max_states, max_rows = dp
+            nb = ks.load().ks_dp_scratch_bytes(self.h, max_states, max_rows)
+            scratch = torch.empty(nb + 256, dtype=torch.uint8, device=self.workspace.device)
+            p.policy = 3
+            p.tpt_max_gamma = int(D)
+            p.dp_scratch = (scratch.data_ptr() + 255) // 256 * 256
+            p.dp_scratch_bytes = nb
+            p.dp_tau = float(tau)
+            p.dp_max_states = int(max_states)
+            p.dp_max_rows = int(max_rows)
+        out = ks.ks_generate_speculative(self.h, p, n_tokens)
+        del scratch
+        return out
 
     def select_dp(self, latency, max_gamma: int, tau: float = 0.5, max_states: int = 128, max_rows: int = 32):
         """Alg. 1 on the current history and the TPT grid over its candidates:

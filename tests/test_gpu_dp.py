@@ -122,3 +122,18 @@ def test_dp_structure_bf16():
     a1 = ar_model.decode_greedy(12)
     a2 = m.decode_greedy(12)
     assert list(a1) == list(a2)
+
+
+@pytest.mark.parametrize("kind", ["tiny", "bf16"])
+def test_dp_policy_in_the_loop_is_lossless(kind):
+    from paper_2602_20217_gb300 import knapspec as ks
+    from paper_2602_20217_gb300.configs import ModelShape, TINY
+    shape = TINY if kind == "tiny" else ModelShape("small-bf16", 2, 512, 8, 2, 128, 1368, 2000, qk_norm=True,
+                                                   dtype="bf16", rope_theta=500000.0)
+    m, seq, p, r_hist = _setup(shape, 31, 12)
+    m2, _, _, _ = _setup(shape, 31, 12)
+    ar = m2.decode_greedy(40)
+    lat = ks.latency(1, units=np.array([2, 1] * shape.n_layers, np.int32))
+    out, st, acc = m.generate(40, 3, latency=lat, resolve_every=5, dp=(6, 0.5, 64, 16))
+    assert list(out) == list(ar)
+    assert st.resolves >= 2
