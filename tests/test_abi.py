@@ -98,6 +98,13 @@ def test_error_paths_touch_no_device(lib):
     g, t = C.c_int32(), C.c_double()
     assert lib.ks_select_tpt(None, C.byref(lat), 4, 4, out.ctypes.data, C.byref(g), C.byref(t), None,
                              None) == ks.KS_ERR_INVALID_ARG
+    samp = ks.sampling(0.7, 50, 0.95, 1)
+    assert lib.ks_draft_sample(None, out.ctypes.data, 4, C.byref(samp), 0, None) == ks.KS_ERR_INVALID_ARG
+    assert lib.ks_verify_sample(None, 4, C.byref(samp), 0, C.byref(a), out.ctypes.data,
+                                C.byref(n)) == ks.KS_ERR_INVALID_ARG
+    assert lib.ks_select_dp(None, C.byref(lat), 0.5, 4, 8, 8, None, 0, out.ctypes.data, C.byref(g), C.byref(t),
+                            None, None, None, None) == ks.KS_ERR_INVALID_ARG
+    assert lib.ks_dp_scratch_bytes(None, 8, 8) == 0
 
 
 def test_select_mask_argument_checks(lib):
