@@ -352,20 +352,28 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const AttnArgs a) {
             // (a) scores of this warp's 16 keys, masked; row maxima to smem
             float sc[2][2][4];
 #pragma unroll
-            for (int u = 0; u < 2; ++u) {
-                if (u >= nm) break;
+            for (int u = 0; u < 2; ++u)
 #pragma unroll
                 for (int j = 0; j < 2; ++j) sc[u][j][0] = sc[u][j][1] = sc[u][j][2] = sc[u][j][3] = 0.f;
+            // each K fragment is loaded once and applied to both m-tiles
 #pragma unroll
-                for (int ks = 0; ks < HD / 16; ++ks) {
-                    uint32_t kb[4];
-                    const int mi = lane >> 3;
-                    const int krow = kk + (mi >> 1) * 8 + (lane & 7);
-                    const int kcol = ks * 16 + (mi & 1) * 8;
-                    ldmatrix_x4(kb, Ks + kv_off<HD>(krow, kcol));
-                    mma_bf16(sc[u][0], qf[u][ks][0], qf[u][ks][1], qf[u][ks][2], qf[u][ks][3], kb[0], kb[1]);
-                    mma_bf16(sc[u][1], qf[u][ks][0], qf[u][ks][1], qf[u][ks][2], qf[u][ks][3], kb[2], kb[3]);
+            for (int ks = 0; ks < HD / 16; ++ks) {
+                uint32_t kb[4];
+                const int mi = lane >> 3;
+                const int krow = kk + (mi >> 1) * 8 + (lane & 7);
+                const int kcol = ks * 16 + (mi & 1) * 8;
+                ldmatrix_x4(kb, Ks + kv_off<HD>(krow, kcol));
+#pragma unroll
+                for (int u = 0; u < 2; ++u) {
+                    if (u < nm) {
+                        mma_bf16(sc[u][0], qf[u][ks][0], qf[u][ks][1], qf[u][ks][2], qf[u][ks][3], kb[0], kb[1]);
+                        mma_bf16(sc[u][1], qf[u][ks][0], qf[u][ks][1], qf[u][ks][2], qf[u][ks][3], kb[2], kb[3]);
+                    }
                 }
+            }
+#pragma unroll
+            for (int u = 0; u < 2; ++u) {
+                if (u >= nm) break;
 #pragma unroll
                 for (int hh = 0; hh < 2; ++hh) {
                     float tmax = -INFINITY;
@@ -438,24 +446,33 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const AttnArgs a) {
                         o[u][i][2 * hh + 1] *= alpha[u][hh];
                     }
                 }
+            }
+            // each V fragment is loaded once and applied to both m-tiles
 #pragma unroll
-                for (int kq = 0; kq < KT / 16; ++kq) {
-                    uint32_t pa[4];
-                    {
+            for (int kq = 0; kq < KT / 16; ++kq) {
+                uint32_t pa[2][4];
+#pragma unroll
+                for (int u = 0; u < 2; ++u) {
+                    if (u < nm) {
                         const int mi = lane >> 3;
                         const int row = (mi & 1) * 8 + (lane & 7);
                         const int col = kq * 16 + (mi >> 1) * 8;
-                        ldmatrix_x4(pa, &Ps[u][row * PP + col]);
+                        ldmatrix_x4(pa[u], &Ps[u][row * PP + col]);
                     }
+                }
 #pragma unroll
-                    for (int dq = 0; dq < WNT / 2; ++dq) {
-                        uint32_t vb[4];
-                        const int mi = lane >> 3;
-                        const int vrow = kq * 16 + (mi & 1) * 8 + (lane & 7);
-                        const int vcol = warp * WD + dq * 16 + (mi >> 1) * 8;
-                        ldmatrix_x4_trans(vb, Vs + kv_off<HD>(vrow, vcol));
-                        mma_bf16(o[u][2 * dq], pa[0], pa[1], pa[2], pa[3], vb[0], vb[1]);
-                        mma_bf16(o[u][2 * dq + 1], pa[0], pa[1], pa[2], pa[3], vb[2], vb[3]);
+                for (int dq = 0; dq < WNT / 2; ++dq) {
+                    uint32_t vb[4];
+                    const int mi = lane >> 3;
+                    const int vrow = kq * 16 + (mi & 1) * 8 + (lane & 7);
+                    const int vcol = warp * WD + dq * 16 + (mi >> 1) * 8;
+                    ldmatrix_x4_trans(vb, Vs + kv_off<HD>(vrow, vcol));
+#pragma unroll
+                    for (int u = 0; u < 2; ++u) {
+                        if (u < nm) {
+                            mma_bf16(o[u][2 * dq], pa[u][0], pa[u][1], pa[u][2], pa[u][3], vb[0], vb[1]);
+                            mma_bf16(o[u][2 * dq + 1], pa[u][0], pa[u][1], pa[u][2], pa[u][3], vb[2], vb[3]);
+                        }
                     }
                 }
             }
