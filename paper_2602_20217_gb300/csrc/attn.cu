@@ -12,16 +12,18 @@
 //
 // Per CTA: the new rows' K (QK-RMSNorm, RoPE) and V are written to the cache
 // by the CTA whose chunk holds their position; the G x R query vectors are
-// normalised, rotated and pre-scaled by log2(e)/sqrt(hd).  bf16 models: K/V
-// tiles of 64 keys stream through a cp.async ring; for up to two 16-row query
-// tiles at a time the four warps split each tile (warp w: Q K^T for keys
-// 16 w.., P V for head dims w HD/4..) on mma.sync.m16n8k16, with an fp32
-// online softmax in the log2 domain over the whole chunk whose row maxima and
-// sums are combined across warps in warp order.  fp32 models: CUDA-core dot products.  Partials (m, l, o) per
-// (row, query head, chunk) are merged by attn_merge_kernel in a fixed order.
-// bf16 launches use programmatic dependent launch: the attention kernel loads
-// its first tile of old keys before waiting for the projections that produce
-// its queries, and both kernels let their successor launch early.
+// normalised, rotated and pre-scaled by log2(e)/sqrt(hd).  bf16 models: keys
+// sit on the M side of mma.sync.m16n8k16 and each of the four warps streams
+// its own 16-key tiles (every fourth tile of the chunk) through a private
+// cp.async ring, with an fp32 online softmax in the log2 domain per query
+// column and no block barrier in the key loop; P reaches the P V product
+// through registers (movmatrix).  The warps' (m, l, o) are combined in warp
+// order at the end of the chunk.  fp32 models: CUDA-core dot products.
+// Partials (m, l, o) per (row, query head, chunk) are merged by
+// attn_merge_kernel in a fixed order.  bf16 launches use programmatic
+// dependent launch: the attention kernel loads its first tiles of old keys
+// before waiting for the projections that produce its queries, and both
+// kernels let their successor launch early.
 #include "common.cuh"
 #include "internal.h"
 
@@ -29,8 +31,6 @@ namespace ks {
 
 constexpr int kAttnWarps = 4;
 constexpr int kPartPad = 4;  // partial row: m, l, 2 pad, o[hd] (16-byte aligned o)
-constexpr int kKeyTile = 64;
-constexpr int kKvStages = 3;   // bf16: K/V tiles in the cp.async ring (two in flight while computing)
 
 // bf16 K/V tiles in shared memory: rows of HD elements, no padding; the
 // 16-byte chunk c of row r is stored at chunk c ^ (r & 7), so the eight rows
@@ -194,16 +194,42 @@ KS_DEV int my_chunk(const AttnArgs& a) {
 }
 
 // ----------------------------------------------------------- bf16 kernel
-// Shared layout (bf16, row pitch hd + 8 elements = 16 B padding):
-//   Qs [mpad][P], then kKvStages stages of { Ks [64][HD], Vs [64][HD] }
-//   (K / V rows unpadded and chunk-swizzled, see kv_off).
-template <int HD>
+// Keys on the M side of the MMA.  Warp w owns keys 16 w .. 16 w + 15 of every
+// 64 keys of the chunk and runs its own online softmax over them, so the key
+// loop needs no block barrier:
+//   S^T (16 keys x 8 NQ query rows)  = K_w Q^T     A = K rows (ldmatrix),
+//                                                   B = Q rows (ldmatrix)
+//   O^T (HD dims x 8 NQ query rows) += V_w^T P^T   A = V (ldmatrix.trans),
+//                                                   B = the S^T accumulator as
+//                                                   bf16, transposed in
+//                                                   registers (movmatrix)
+// A warp's K/V rows stream through its own cp.async ring of kWarpStages
+// 16-key tiles.  At the end of a chunk the four warps' (m, l, O) meet in
+// their ring space and are combined in warp order.  Query rows m = r G + gq
+// are taken in rounds of 8 NQ rows (each round streams the chunk again).
+// Every step of a query row's arithmetic is fixed by the chunk and the key
+// index alone, never by R or by the other rows of the pass.
+constexpr int kWarpKeys = 16;
+constexpr int kWarpStages = 3;
+
+// 8x8 b16 matrix transpose across the warp: the fragment of X becomes the
+// fragment of X^T
+KS_DEV uint32_t movmatrix_trans(uint32_t x) {
+    uint32_t y;
+    asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;\n" : "=r"(y) : "r"(x));
+    return y;
+}
+
+template <int HD, int NQ>
 __global__ void __launch_bounds__(128) attn_bf16_kernel(const AttnArgs a) {
     if (a.stop && *a.stop) return;   // a draft pass after the dynamic exit
     constexpr int NPL = HD / 32;
-    constexpr int P = HD + 8;
-    constexpr int NDT = HD / 8;  // dim tiles of 8
-    constexpr int KT = kKeyTile;
+    constexpr int P = HD + 8;          // Qs row pitch (bf16)
+    constexpr int KD = HD / 16;        // k-steps of K Q^T = dim tiles of V^T P^T
+    constexpr int QR = 8 * NQ;         // query rows per round
+    constexpr int RING = kWarpStages * 2 * kWarpKeys * HD;   // a warp's ring (bf16 elements)
+    constexpr int OP = HD + 4;         // pitch of a query row in the combine area (fp32)
+    static_assert(QR * (OP + 2) * 4 <= RING * 2, "combine area exceeds the warp's ring");
     extern __shared__ __align__(16) unsigned char smem[];
 
     const int h = blockIdx.x, c = my_chunk(a);
@@ -211,14 +237,14 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const AttnArgs a) {
     const int g = lane >> 2, t = lane & 3;
     const int G = a.hq / a.hk;
     const int M = G * a.R;
-    const int mtiles = (M + 15) >> 4;
-    const int mpad = mtiles * 16;
+    const int rounds = (M + QR - 1) / QR;
     const int cs = attn_chunk_start(c);
     const int ce = min(attn_chunk_start(c + 1), a.p0 + a.R);  // valid keys [cs, ce)
-    const int ntiles = (ce - cs + KT - 1) / KT;
+    const int nwt = (ce - cs + kWarpKeys - 1) / kWarpKeys;    // 16-key tiles of the chunk
+    const int my_n = nwt > warp ? (nwt - warp + kAttnWarps - 1) / kAttnWarps : 0;  // tiles warp, warp + 4, ..
 
     __nv_bfloat16* Qs = reinterpret_cast<__nv_bfloat16*>(smem);
-    __nv_bfloat16* KV = Qs + (size_t)mpad * P;  // stage s: K at KV + s*2*KT*HD, V after it
+    __nv_bfloat16* ring = Qs + QR * P + warp * RING;
 
     // The merge kernel may launch now; it reads the partials only after this
     // grid completes.
@@ -226,13 +252,15 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const AttnArgs a) {
 
     const __nv_bfloat16* kg = reinterpret_cast<const __nv_bfloat16*>(a.kcache) + (size_t)h * a.max_seq * HD;
     const __nv_bfloat16* vg = reinterpret_cast<const __nv_bfloat16*>(a.vcache) + (size_t)h * a.max_seq * HD;
-    constexpr int CPR = HD / 8;  // 16-byte pieces per row
-    auto load_tile = [&](int ti) {
-        __nv_bfloat16* Ks = KV + (size_t)(ti % kKvStages) * 2 * KT * HD;
-        __nv_bfloat16* Vs = Ks + (size_t)KT * HD;
-        const int k0 = cs + ti * KT;
-        for (int i = tid; i < KT * CPR; i += blockDim.x) {
-            const int row = i / CPR, col = (i - row * CPR) * 8;
+    // this warp's i-th tile -> stage i % kWarpStages
+    auto load_tile = [&](int i) {
+        __nv_bfloat16* Ks = ring + (i % kWarpStages) * 2 * kWarpKeys * HD;
+        __nv_bfloat16* Vs = Ks + kWarpKeys * HD;
+        const int k0 = cs + (warp + kAttnWarps * i) * kWarpKeys;
+        constexpr int CPR = HD / 8;   // 16-byte pieces per row
+#pragma unroll
+        for (int j = lane; j < kWarpKeys * CPR; j += 32) {
+            const int row = j / CPR, col = (j - row * CPR) * 8;
             const bool ok = k0 + row < ce;
             const size_t off = ok ? (size_t)(k0 + row) * HD + col : 0;
             cp_async16(Ks + kv_off<HD>(row, col), kg + off, ok);
@@ -240,264 +268,219 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const AttnArgs a) {
         }
         cp_async_commit();
     };
-    // Keys before p0 were written by earlier launches (complete before the
-    // projections that precede this kernel could start), so the first tiles
-    // of old keys go out before waiting for the projections.
-    const int pre = min(kKvStages - 1, ntiles);   // tiles loaded ahead of the loop
+    auto tile_old = [&](int i) { return cs + (warp + kAttnWarps * i + 1) * kWarpKeys <= a.p0; };
+    // Keys before p0 were written by earlier launches, so this warp's first
+    // tiles of old keys go out before waiting for the projections.
+    const int pre = min(kWarpStages - 1, my_n);
     int loaded = 0;
-    while (loaded < pre && cs + (loaded + 1) * KT <= a.p0) load_tile(loaded++);
+    while (loaded < pre && tile_old(loaded)) load_tile(loaded++);
     asm volatile("griddepcontrol.wait;" ::: "memory");
 
-    // 1. new K/V rows of this chunk -> cache (generic stores, then barrier)
+    // new K/V rows of this chunk -> cache (generic stores, then barrier)
     write_new_kv<__nv_bfloat16, NPL>(a, h, cs, ce);
     __syncthreads();
     while (loaded < pre) load_tile(loaded++);
 
-    // 2. queries: m = r * G + gq, scaled into the log2 domain, bf16
     const float qscale = kLog2e * rsqrtf((float)HD);
     const __nv_bfloat16* qn = reinterpret_cast<const __nv_bfloat16*>(a.q_norm);
-    constexpr int QB = 4;
-    for (int m0 = warp * QB; m0 < mpad; m0 += kAttnWarps * QB) {
-        const float* src[QB];
-        bool valid[QB];
-        int pos[QB];
-#pragma unroll
-        for (int j = 0; j < QB; ++j) {
-            const int m = m0 + j;
-            valid[j] = m < M;
-            const int r = valid[j] ? m / G : 0, gq = valid[j] ? m - r * G : 0;
-            src[j] = a.qkv + (size_t)r * a.qkv_ld + (h * G + gq) * HD;
-            pos[j] = a.p0 + r;
+    for (int rd = 0; rd < rounds; ++rd) {
+        const int q0 = rd * QR;   // first query row of the round
+        if (rd > 0) {             // the rings (and combine areas) are free again
+            __syncthreads();
+            loaded = 0;
+            while (loaded < pre) load_tile(loaded++);
         }
-        float q[QB][NPL];
-        head_vectors<__nv_bfloat16, NPL, QB>(src, valid, pos, qn, a.eps, a.rope, q);
+        // queries of the round: m = q0 + row, scaled into the log2 domain, bf16
+        constexpr int QB = 4;
+        for (int r0 = warp * QB; r0 < QR; r0 += kAttnWarps * QB) {
+            const float* src[QB];
+            bool valid[QB];
+            int pos[QB];
 #pragma unroll
-        for (int j = 0; j < QB; ++j) {
-            const int m = m0 + j;
-            if (m >= mpad) continue;
-#pragma unroll
-            for (int i = 0; i < NPL; ++i)
-                Qs[m * P + lane + 32 * i] = __float2bfloat16_rn(valid[j] ? q[j][i] * qscale : 0.f);
-        }
-    }
-
-    // 3. rounds of up to two m-tiles.  In a round the four warps split every
-    //    64-key tile: warp w scores keys 16 w .. 16 w + 15 (Q K^T) and
-    //    accumulates head dims w HD/4 .. (w + 1) HD/4 of P V over all 64 keys.
-    //    Row maxima and row sums meet in shared memory and are combined in
-    //    warp order, so a row's arithmetic is the same for every R.
-    constexpr int WD = HD / kAttnWarps;   // head dims per warp
-    constexpr int WNT = WD / 8;           // n8 tiles of P V per warp
-    constexpr int PP = KT + 8;            // pitch of the probability tile
-    __shared__ __align__(16) __nv_bfloat16 Ps[2][16 * PP];
-    __shared__ float red_max[2][kAttnWarps][16];
-    __shared__ float red_sum[2][kAttnWarps][16];
-    for (int mt0 = 0; mt0 < mtiles; mt0 += 2) {
-        const int nm = min(2, mtiles - mt0);
-        if (mt0 > 0)   // a new round streams the chunk again
-            for (int j = 0; j < pre; ++j) load_tile(j);
-        uint32_t qf[2][HD / 16][4];
-        int rpos[2][2];
-        float o[2][WNT][4];
-        float mrow[2][2], lrow[2][2];
-#pragma unroll
-        for (int u = 0; u < 2; ++u)
-#pragma unroll
-            for (int hh = 0; hh < 2; ++hh) {
-                mrow[u][hh] = -INFINITY;
-                lrow[u][hh] = 0.f;
-                rpos[u][hh] = -1;
+            for (int j = 0; j < QB; ++j) {
+                const int m = q0 + r0 + j;
+                valid[j] = m < M;
+                const int r = valid[j] ? m / G : 0, gq = valid[j] ? m - r * G : 0;
+                src[j] = a.qkv + (size_t)r * a.qkv_ld + (h * G + gq) * HD;
+                pos[j] = a.p0 + r;
             }
+            float q[QB][NPL];
+            head_vectors<__nv_bfloat16, NPL, QB>(src, valid, pos, qn, a.eps, a.rope, q);
 #pragma unroll
-        for (int u = 0; u < 2; ++u)
+            for (int j = 0; j < QB; ++j) {
+                if (r0 + j >= QR) continue;
 #pragma unroll
-            for (int i = 0; i < WNT; ++i) o[u][i][0] = o[u][i][1] = o[u][i][2] = o[u][i][3] = 0.f;
-        bool qloaded = false;
+                for (int i = 0; i < NPL; ++i)
+                    Qs[(r0 + j) * P + lane + 32 * i] = __float2bfloat16_rn(valid[j] ? q[j][i] * qscale : 0.f);
+            }
+        }
+        __syncthreads();   // Qs complete
+        // Q^T fragments (B operand): query tile j = rows 8 j .., k-step ks
+        uint32_t qf[NQ][KD][2];
+#pragma unroll
+        for (int j = 0; j < NQ; ++j)
+#pragma unroll
+            for (int ks = 0; ks < KD; ks += 2) {
+                uint32_t r4[4];
+                ldmatrix_x4(r4, Qs + (8 * j + (lane & 7)) * P + ks * 16 + (lane >> 3) * 8);
+                qf[j][ks][0] = r4[0];
+                qf[j][ks][1] = r4[1];
+                qf[j][ks + 1][0] = r4[2];
+                qf[j][ks + 1][1] = r4[3];
+            }
+        // this thread's query columns: 8 j + 2 t + e; padding rows see no key
+        int qpos[NQ][2];
+#pragma unroll
+        for (int j = 0; j < NQ; ++j)
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+                const int m = q0 + 8 * j + 2 * t + e;
+                qpos[j][e] = m < M ? a.p0 + m / G : -1;
+            }
+        float o[KD][NQ][4];          // O^T: dims 16 d + g (+ 8), query columns 8 j + 2 t (+ 1)
+        float mcol[NQ][2], lsum[NQ][2];
+#pragma unroll
+        for (int j = 0; j < NQ; ++j) {
+#pragma unroll
+            for (int d = 0; d < KD; ++d) o[d][j][0] = o[d][j][1] = o[d][j][2] = o[d][j][3] = 0.f;
+            mcol[j][0] = mcol[j][1] = -INFINITY;
+            lsum[j][0] = lsum[j][1] = 0.f;   // this thread's keys g, g + 8 only
+        }
 
-        for (int ti = 0; ti < ntiles; ++ti) {
-            // tile ti + kKvStages - 1 goes into the slot tile ti - 1 used
-            if (ti + kKvStages - 1 < ntiles) {
-                load_tile(ti + kKvStages - 1);
-                cp_async_wait<kKvStages - 1>();
-            } else if (ti + 1 < ntiles) {
-                cp_async_wait<1>();   // tile ti + 1 may stay in flight
+        for (int i = 0; i < my_n; ++i) {
+            // tile i + kWarpStages - 1 goes into the stage tile i - 1 used
+            if (i + kWarpStages - 1 < my_n) {
+                load_tile(i + kWarpStages - 1);
+                cp_async_wait<kWarpStages - 1>();
+            } else if (i + 1 < my_n) {
+                cp_async_wait<1>();
             } else {
                 cp_async_wait<0>();
             }
-            __syncthreads();  // tile ti (and, first time, Qs) visible
-            if (!qloaded) {
+            __syncwarp();   // every lane's copies of tile i are visible
+            const __nv_bfloat16* Ks = ring + (i % kWarpStages) * 2 * kWarpKeys * HD;
+            const __nv_bfloat16* Vs = Ks + kWarpKeys * HD;
+            const int k0 = cs + (warp + kAttnWarps * i) * kWarpKeys;
+            // (a) S^T = K Q^T for this warp's 16 keys
+            float s[NQ][4];
 #pragma unroll
-                for (int u = 0; u < 2; ++u) {
-                    if (u >= nm) break;
-                    const int mt = mt0 + u;
+            for (int j = 0; j < NQ; ++j) s[j][0] = s[j][1] = s[j][2] = s[j][3] = 0.f;
 #pragma unroll
-                    for (int ks = 0; ks < HD / 16; ++ks) {
-                        const int mi = lane >> 3;
-                        const int row = mt * 16 + (mi & 1) * 8 + (lane & 7);
-                        const int col = ks * 16 + (mi >> 1) * 8;
-                        ldmatrix_x4(qf[u][ks], Qs + row * P + col);
-                    }
+            for (int ks = 0; ks < KD; ++ks) {
+                uint32_t ka[4];
+                ldmatrix_x4(ka, Ks + kv_off<HD>((lane & 7) + ((lane >> 3) & 1) * 8, ks * 16 + (lane >> 4) * 8));
 #pragma unroll
-                    for (int hh = 0; hh < 2; ++hh) {
-                        const int m = mt * 16 + g + 8 * hh;
-                        rpos[u][hh] = (m < M) ? a.p0 + m / G : -1;  // padding rows see no key
-                    }
-                }
-                qloaded = true;
+                for (int j = 0; j < NQ; ++j) mma_bf16(s[j], ka[0], ka[1], ka[2], ka[3], qf[j][ks][0], qf[j][ks][1]);
             }
-            const __nv_bfloat16* Ks = KV + (size_t)(ti % kKvStages) * 2 * KT * HD;
-            const __nv_bfloat16* Vs = Ks + (size_t)KT * HD;
-            const int kk = 16 * warp;               // this warp's keys in the tile
-            const int kbase = cs + ti * KT + kk;
-            // (a) scores of this warp's 16 keys, masked; row maxima to smem
-            float sc[2][2][4];
+            // (b) mask, online softmax per query column over this warp's keys
+            const int key0 = k0 + g, key1 = k0 + g + 8;
+            uint32_t pb[NQ][2];
 #pragma unroll
-            for (int u = 0; u < 2; ++u)
+            for (int j = 0; j < NQ; ++j) {
 #pragma unroll
-                for (int j = 0; j < 2; ++j) sc[u][j][0] = sc[u][j][1] = sc[u][j][2] = sc[u][j][3] = 0.f;
-            // each K fragment is loaded once and applied to both m-tiles
-#pragma unroll
-            for (int ks = 0; ks < HD / 16; ++ks) {
-                uint32_t kb[4];
-                const int mi = lane >> 3;
-                const int krow = kk + (mi >> 1) * 8 + (lane & 7);
-                const int kcol = ks * 16 + (mi & 1) * 8;
-                ldmatrix_x4(kb, Ks + kv_off<HD>(krow, kcol));
-#pragma unroll
-                for (int u = 0; u < 2; ++u) {
-                    if (u < nm) {
-                        mma_bf16(sc[u][0], qf[u][ks][0], qf[u][ks][1], qf[u][ks][2], qf[u][ks][3], kb[0], kb[1]);
-                        mma_bf16(sc[u][1], qf[u][ks][0], qf[u][ks][1], qf[u][ks][2], qf[u][ks][3], kb[2], kb[3]);
-                    }
-                }
-            }
-#pragma unroll
-            for (int u = 0; u < 2; ++u) {
-                if (u >= nm) break;
-#pragma unroll
-                for (int hh = 0; hh < 2; ++hh) {
-                    float tmax = -INFINITY;
-#pragma unroll
-                    for (int j = 0; j < 2; ++j)
-#pragma unroll
-                        for (int e = 0; e < 2; ++e) {
-                            const int key = kbase + j * 8 + 2 * t + e;
-                            float& v = sc[u][j][2 * hh + e];
-                            if (key > rpos[u][hh] || key >= ce) v = -INFINITY;
-                            tmax = fmaxf(tmax, v);
-                        }
-                    tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 1));
-                    tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 2));
-                    if (t == 0) red_max[u][warp][g + 8 * hh] = tmax;
-                }
-            }
-            __syncthreads();
-            // (b) the tile's row maximum, probabilities to smem, row sums to smem
-            float alpha[2][2];
-#pragma unroll
-            for (int u = 0; u < 2; ++u) {
-                if (u >= nm) break;
-#pragma unroll
-                for (int hh = 0; hh < 2; ++hh) {
-                    const int row = g + 8 * hh;
-                    const float tile_max = fmaxf(fmaxf(red_max[u][0][row], red_max[u][1][row]),
-                                                 fmaxf(red_max[u][2][row], red_max[u][3][row]));
-                    const float mnew = fmaxf(mrow[u][hh], tile_max);
-                    float psum = 0.f;
-                    if (mnew == -INFINITY) {
-                        alpha[u][hh] = 1.f;
-#pragma unroll
-                        for (int j = 0; j < 2; ++j) sc[u][j][2 * hh] = sc[u][j][2 * hh + 1] = 0.f;
+                for (int e = 0; e < 2; ++e) {
+                    float& va = s[j][e];
+                    float& vb = s[j][2 + e];
+                    if (key0 > qpos[j][e] || key0 >= ce) va = -INFINITY;
+                    if (key1 > qpos[j][e] || key1 >= ce) vb = -INFINITY;
+                    float tmax = fmaxf(va, vb);
+                    tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 4));
+                    tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 8));
+                    tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 16));
+                    const float mnew = fmaxf(mcol[j][e], tmax);
+                    float alpha = 1.f;
+                    if (mnew == -INFINITY) {   // no key of this column seen yet
+                        va = vb = 0.f;
                     } else {
-                        alpha[u][hh] = exp2f(mrow[u][hh] - mnew);
-#pragma unroll
-                        for (int j = 0; j < 2; ++j)
-#pragma unroll
-                            for (int e = 0; e < 2; ++e) {
-                                float& v = sc[u][j][2 * hh + e];
-                                v = exp2f(v - mnew);
-                                psum += v;
-                            }
+                        alpha = exp2f(mcol[j][e] - mnew);
+                        va = exp2f(va - mnew);
+                        vb = exp2f(vb - mnew);
                     }
-                    mrow[u][hh] = mnew;
-                    psum += __shfl_xor_sync(0xffffffffu, psum, 1);
-                    psum += __shfl_xor_sync(0xffffffffu, psum, 2);
-                    if (t == 0) red_sum[u][warp][row] = psum;
+                    mcol[j][e] = mnew;
+                    lsum[j][e] = lsum[j][e] * alpha + (va + vb);
 #pragma unroll
-                    for (int j = 0; j < 2; ++j)
-                        *reinterpret_cast<uint32_t*>(&Ps[u][row * PP + kk + 8 * j + 2 * t]) =
-                            pack_bf16(sc[u][j][2 * hh], sc[u][j][2 * hh + 1]);
+                    for (int d = 0; d < KD; ++d) {
+                        o[d][j][e] *= alpha;
+                        o[d][j][2 + e] *= alpha;
+                    }
                 }
+                // P^T (keys x queries) as the B operand: transposed S^T fragments
+                pb[j][0] = movmatrix_trans(pack_bf16(s[j][0], s[j][1]));
+                pb[j][1] = movmatrix_trans(pack_bf16(s[j][2], s[j][3]));
             }
-            __syncthreads();
-            // (c) l and o rescaled; O += P V over the 64 keys for this warp's dims
+            // (c) O^T += V^T P^T over this warp's 16 keys
 #pragma unroll
-            for (int u = 0; u < 2; ++u) {
-                if (u >= nm) break;
+            for (int d = 0; d < KD; ++d) {
+                uint32_t va[4];
+                const int mi = lane >> 3;
+                ldmatrix_x4_trans(va, Vs + kv_off<HD>((lane & 7) + (mi >> 1) * 8, d * 16 + (mi & 1) * 8));
 #pragma unroll
-                for (int hh = 0; hh < 2; ++hh) {
-                    const int row = g + 8 * hh;
-                    const float tsum = ((red_sum[u][0][row] + red_sum[u][1][row]) + red_sum[u][2][row]) +
-                                       red_sum[u][3][row];
-                    lrow[u][hh] = lrow[u][hh] * alpha[u][hh] + tsum;
-#pragma unroll
-                    for (int i = 0; i < WNT; ++i) {
-                        o[u][i][2 * hh] *= alpha[u][hh];
-                        o[u][i][2 * hh + 1] *= alpha[u][hh];
-                    }
-                }
+                for (int j = 0; j < NQ; ++j) mma_bf16(o[d][j], va[0], va[1], va[2], va[3], pb[j][0], pb[j][1]);
             }
-            // each V fragment is loaded once and applied to both m-tiles
-#pragma unroll
-            for (int kq = 0; kq < KT / 16; ++kq) {
-                uint32_t pa[2][4];
-#pragma unroll
-                for (int u = 0; u < 2; ++u) {
-                    if (u < nm) {
-                        const int mi = lane >> 3;
-                        const int row = (mi & 1) * 8 + (lane & 7);
-                        const int col = kq * 16 + (mi >> 1) * 8;
-                        ldmatrix_x4(pa[u], &Ps[u][row * PP + col]);
-                    }
-                }
-#pragma unroll
-                for (int dq = 0; dq < WNT / 2; ++dq) {
-                    uint32_t vb[4];
-                    const int mi = lane >> 3;
-                    const int vrow = kq * 16 + (mi & 1) * 8 + (lane & 7);
-                    const int vcol = warp * WD + dq * 16 + (mi >> 1) * 8;
-                    ldmatrix_x4_trans(vb, Vs + kv_off<HD>(vrow, vcol));
-#pragma unroll
-                    for (int u = 0; u < 2; ++u) {
-                        if (u < nm) {
-                            mma_bf16(o[u][2 * dq], pa[u][0], pa[u][1], pa[u][2], pa[u][3], vb[0], vb[1]);
-                            mma_bf16(o[u][2 * dq + 1], pa[u][0], pa[u][1], pa[u][2], pa[u][3], vb[2], vb[3]);
-                        }
-                    }
-                }
-            }
-            __syncthreads();  // everyone is done with tile ti (and Ps, red_*) before reuse
+            __syncwarp();   // every lane is done with the stage before it is refilled
         }
-        // this chunk's partials: m and l by warp 0, each warp its dims of o
+        // (d) this warp's column sums, then (m, l, O^T) into its ring space
 #pragma unroll
-        for (int u = 0; u < 2; ++u) {
-            if (u >= nm) break;
+        for (int j = 0; j < NQ; ++j)
 #pragma unroll
-            for (int hh = 0; hh < 2; ++hh) {
-                const int m = (mt0 + u) * 16 + g + 8 * hh;
-                if (m >= M) continue;
-                const int r = m / G, gq = m - r * G;
-                float* dst = a.part + (((size_t)r * a.hq + h * G + gq) * a.n_chunks_max + c) * (HD + kPartPad);
-                if (warp == 0 && t == 0) {
-                    dst[0] = mrow[u][hh];
-                    dst[1] = lrow[u][hh];
+            for (int e = 0; e < 2; ++e) {
+                float l = lsum[j][e];
+                l += __shfl_xor_sync(0xffffffffu, l, 4);
+                l += __shfl_xor_sync(0xffffffffu, l, 8);
+                l += __shfl_xor_sync(0xffffffffu, l, 16);
+                lsum[j][e] = l;
+            }
+        float* cm = reinterpret_cast<float*>(ring);   // [QR] m, [QR] l, [QR][OP] o
+        float* cl = cm + QR;
+        float* co = cl + QR;
+#pragma unroll
+        for (int j = 0; j < NQ; ++j)
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+                const int q = 8 * j + 2 * t + e;
+                if (g == 0) {
+                    cm[q] = mcol[j][e];
+                    cl[q] = lsum[j][e];
                 }
 #pragma unroll
-                for (int i = 0; i < WNT; ++i) {
-                    dst[kPartPad + warp * WD + i * 8 + 2 * t] = o[u][i][2 * hh];
-                    dst[kPartPad + warp * WD + i * 8 + 2 * t + 1] = o[u][i][2 * hh + 1];
+                for (int d = 0; d < KD; ++d) {
+                    co[q * OP + 16 * d + g] = o[d][j][e];
+                    co[q * OP + 16 * d + g + 8] = o[d][j][2 + e];
                 }
             }
+        __syncthreads();
+        // (e) the four warps combined in warp order -> this chunk's partials:
+        //     per query row the chunk maximum, each warp's scale factor and
+        //     the sum l (one thread per row), then O element by element
+        const int nq = min(QR, M - q0);
+        const float* wsum = reinterpret_cast<const float*>(Qs + QR * P);   // warp w at w * RING * 2 floats
+        constexpr int WF = RING / 2;                                         // floats per warp's ring
+        float* fac = reinterpret_cast<float*>(Qs);   // [kAttnWarps][QR] (Qs is free until the next round)
+        if (tid < nq) {
+            const int q = tid;
+            float gm = -INFINITY;
+#pragma unroll
+            for (int w = 0; w < kAttnWarps; ++w) gm = fmaxf(gm, wsum[w * WF + q]);
+            float L = 0.f;
+#pragma unroll
+            for (int w = 0; w < kAttnWarps; ++w) {
+                const float f = gm == -INFINITY ? 0.f : exp2f(wsum[w * WF + q] - gm);   // 0: a warp that saw no key
+                fac[w * QR + q] = f;
+                L += wsum[w * WF + QR + q] * f;
+            }
+            const int m = q0 + q, r = m / G, gq = m - r * G;
+            float* dst = a.part + (((size_t)r * a.hq + h * G + gq) * a.n_chunks_max + c) * (HD + kPartPad);
+            dst[0] = gm;
+            dst[1] = L;
+        }
+        __syncthreads();
+        for (int idx = tid; idx < nq * HD; idx += blockDim.x) {
+            const int q = idx / HD, dim = idx - q * HD;
+            float O = 0.f;
+#pragma unroll
+            for (int w = 0; w < kAttnWarps; ++w) O += wsum[w * WF + 2 * QR + q * OP + dim] * fac[w * QR + q];
+            const int m = q0 + q, r = m / G, gq = m - r * G;
+            a.part[(((size_t)r * a.hq + h * G + gq) * a.n_chunks_max + c) * (HD + kPartPad) + kPartPad + dim] = O;
         }
     }
 }
@@ -638,9 +621,9 @@ __global__ void __launch_bounds__(128) attn_merge_kernel(const AttnArgs a) {
 }
 
 // --------------------------------------------------------------- launchers
-static size_t attn_bf16_smem(int HD, int mpad) {
-    const int P = HD + 8;
-    return sizeof(__nv_bfloat16) * ((size_t)mpad * P + (size_t)kKvStages * 2 * kKeyTile * HD);
+static size_t attn_bf16_smem(int HD, int NQ) {
+    return sizeof(__nv_bfloat16) *
+           ((size_t)8 * NQ * (HD + 8) + (size_t)kAttnWarps * kWarpStages * 2 * kWarpKeys * HD);
 }
 
 cudaError_t launch_attention(int dtype, const AttnArgs& a, cudaStream_t s) {
@@ -648,9 +631,10 @@ cudaError_t launch_attention(int dtype, const AttnArgs& a, cudaStream_t s) {
     if (nch > a.n_chunks_max || a.p0 + a.R > a.max_seq) return cudaErrorInvalidValue;
     dim3 grid(a.hk, nch);
     if (dtype == 1) {
+        // query rows per round: 8 NQ (rows beyond 24 take further rounds)
         const int M = (a.hq / a.hk) * a.R;
-        const int mpad = ((M + 15) / 16) * 16;
-        const size_t smem = attn_bf16_smem(a.hd, mpad);
+        const int NQ = M <= 8 ? 1 : M <= 16 ? 2 : 3;
+        const size_t smem = attn_bf16_smem(a.hd, NQ);
         auto run = [&](auto kern) -> cudaError_t {
             cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
             if (e != cudaSuccess) return e;
@@ -666,8 +650,10 @@ cudaError_t launch_attention(int dtype, const AttnArgs& a, cudaStream_t s) {
             cfg.numAttrs = 1;
             return cudaLaunchKernelEx(&cfg, kern, a);
         };
-        if (a.hd == 128) return run(attn_bf16_kernel<128>);
-        if (a.hd == 64) return run(attn_bf16_kernel<64>);
+        if (a.hd == 128) return NQ == 1 ? run(attn_bf16_kernel<128, 1>)
+                              : NQ == 2 ? run(attn_bf16_kernel<128, 2>) : run(attn_bf16_kernel<128, 3>);
+        if (a.hd == 64) return NQ == 1 ? run(attn_bf16_kernel<64, 1>)
+                             : NQ == 2 ? run(attn_bf16_kernel<64, 2>) : run(attn_bf16_kernel<64, 3>);
         return cudaErrorInvalidValue;
     }
     const size_t smem = sizeof(float) * kAttnWarps * ((size_t)a.hd + 2048);
