@@ -277,8 +277,10 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const AttnArgs a) {
     asm volatile("griddepcontrol.wait;" ::: "memory");
 
     // new K/V rows of this chunk -> cache (generic stores, then barrier)
-    write_new_kv<__nv_bfloat16, NPL>(a, h, cs, ce);
-    __syncthreads();
+    if (ce > a.p0) {
+        write_new_kv<__nv_bfloat16, NPL>(a, h, cs, ce);
+        __syncthreads();
+    }
     while (loaded < pre) load_tile(loaded++);
 
     const float qscale = kLog2e * rsqrtf((float)HD);
@@ -291,7 +293,8 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const AttnArgs a) {
             while (loaded < pre) load_tile(loaded++);
         }
         // queries of the round: m = q0 + row, scaled into the log2 domain, bf16
-        constexpr int QB = 4;
+        // (2 NQ rows per warp: one pass over the round's rows)
+        constexpr int QB = 2 * NQ;
         for (int r0 = warp * QB; r0 < QR; r0 += kAttnWarps * QB) {
             const float* src[QB];
             bool valid[QB];
@@ -315,10 +318,12 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const AttnArgs a) {
             }
         }
         __syncthreads();   // Qs complete
-        // Q^T fragments (B operand): query tile j = rows 8 j .., k-step ks
-        uint32_t qf[NQ][KD][2];
+        // Q^T fragments (B operand): query tile j = rows 8 j .., k-step ks;
+        // held in registers for up to two query tiles, else read from Qs
+        constexpr bool kQReg = NQ <= 2;
+        uint32_t qf[kQReg ? NQ : 1][KD][2];
 #pragma unroll
-        for (int j = 0; j < NQ; ++j)
+        for (int j = 0; j < (kQReg ? NQ : 0); ++j)
 #pragma unroll
             for (int ks = 0; ks < KD; ks += 2) {
                 uint32_t r4[4];
@@ -366,11 +371,25 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const AttnArgs a) {
 #pragma unroll
             for (int j = 0; j < NQ; ++j) s[j][0] = s[j][1] = s[j][2] = s[j][3] = 0.f;
 #pragma unroll
-            for (int ks = 0; ks < KD; ++ks) {
-                uint32_t ka[4];
-                ldmatrix_x4(ka, Ks + kv_off<HD>((lane & 7) + ((lane >> 3) & 1) * 8, ks * 16 + (lane >> 4) * 8));
+            for (int ks = 0; ks < KD; ks += 2) {
+                uint32_t ka[2][4];
 #pragma unroll
-                for (int j = 0; j < NQ; ++j) mma_bf16(s[j], ka[0], ka[1], ka[2], ka[3], qf[j][ks][0], qf[j][ks][1]);
+                for (int u = 0; u < 2; ++u)
+                    ldmatrix_x4(ka[u], Ks + kv_off<HD>((lane & 7) + ((lane >> 3) & 1) * 8, (ks + u) * 16 + (lane >> 4) * 8));
+#pragma unroll
+                for (int j = 0; j < NQ; ++j) {
+                    uint32_t b[4];
+                    if constexpr (kQReg) {
+                        b[0] = qf[j][ks][0];
+                        b[1] = qf[j][ks][1];
+                        b[2] = qf[j][ks + 1][0];
+                        b[3] = qf[j][ks + 1][1];
+                    } else {
+                        ldmatrix_x4(b, Qs + (8 * j + (lane & 7)) * P + ks * 16 + (lane >> 3) * 8);
+                    }
+                    mma_bf16(s[j], ka[0][0], ka[0][1], ka[0][2], ka[0][3], b[0], b[1]);
+                    mma_bf16(s[j], ka[1][0], ka[1][1], ka[1][2], ka[1][3], b[2], b[3]);
+                }
             }
             // (b) mask, online softmax per query column over this warp's keys
             const int key0 = k0 + g, key1 = k0 + g + 8;
@@ -474,13 +493,22 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const AttnArgs a) {
             dst[1] = L;
         }
         __syncthreads();
-        for (int idx = tid; idx < nq * HD; idx += blockDim.x) {
-            const int q = idx / HD, dim = idx - q * HD;
-            float O = 0.f;
+        constexpr int HV = HD / 4;   // float4 pieces of a row
+        for (int idx = tid; idx < nq * HV; idx += blockDim.x) {
+            const int q = idx / HV, d4 = (idx - q * HV) * 4;
+            float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-            for (int w = 0; w < kAttnWarps; ++w) O += wsum[w * WF + 2 * QR + q * OP + dim] * fac[w * QR + q];
+            for (int w = 0; w < kAttnWarps; ++w) {
+                const float4 v = *reinterpret_cast<const float4*>(wsum + w * WF + 2 * QR + q * OP + d4);
+                const float f = fac[w * QR + q];
+                O.x += v.x * f;
+                O.y += v.y * f;
+                O.z += v.z * f;
+                O.w += v.w * f;
+            }
             const int m = q0 + q, r = m / G, gq = m - r * G;
-            a.part[(((size_t)r * a.hq + h * G + gq) * a.n_chunks_max + c) * (HD + kPartPad) + kPartPad + dim] = O;
+            *reinterpret_cast<float4*>(a.part + (((size_t)r * a.hq + h * G + gq) * a.n_chunks_max + c) * (HD + kPartPad) +
+                                       kPartPad + d4) = O;
         }
     }
 }
