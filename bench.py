@@ -245,7 +245,12 @@ def gpu_arm(args):
     t_prefill = prefill()
     progress("prefill done; latency model")
     split = [k for name, k in ks.KLASS.items() if name != "chain"]   # one projection per launch
-    for k in split:
+    for k in split:                  # untimed first launches of every kernel in that mode
+        ks.ks_kernel_timing(h, k, True)
+    model.decode_greedy(3)
+    rewind()
+    for k in split:                  # disabling resets the class's counters; re-enable to time
+        ks.ks_kernel_timing(h, k, False)
         ks.ks_kernel_timing(h, k, True)
     model.decode_greedy(8)
     kt = {name: ks.ks_kernel_time(h, k) for name, k in ks.KLASS.items() if name != "chain"}
@@ -398,6 +403,17 @@ def gpu_arm(args):
         # dominant kernel: the chained projections; algorithmic bytes = the
         # weight bytes of the projections each launch ran
         achieved = ch_bytes / (ch_ms * 1e-3) / 1e9 if ch_ms > 0 else 0.0
+        # second kernel: split-KV attention of the greedy passes that calibrated
+        # the latency model (R = 1, contexts prompt_len .. prompt_len + 7, CUDA
+        # events around each launch); algorithmic bytes = the layer's K and V
+        # up to the row's position
+        n_ctx = wl.prompt_len + 4.5
+        kv_bytes = 2.0 * sh.n_kv_heads * n_ctx * sh.head_dim * (2 if sh.dtype == "bf16" else 4)
+        t_attn = per("attn") * 1e-3
+        attn_roof = {"bound": "hbm", "achieved": kv_bytes / t_attn / 1e9 if t_attn > 0 else 0.0, "peak": peak,
+                     "unit": "GB/s", "frac": (kv_bytes / t_attn / 1e9) / peak if t_attn > 0 else 0.0,
+                     "kernel": "attn_bf16_kernel (R = 1, one launch per layer)", "bytes_per_launch": kv_bytes,
+                     "us_per_launch": per("attn") * 1e3, "context": n_ctx}
         line = {
             "metric": METRIC, "value": tok_all / (ms_max * 1e-3), "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_max / args.steps,
@@ -431,6 +447,7 @@ def gpu_arm(args):
                          "launches_timed": ch_n, "bytes_per_launch": ch_bytes / max(1, ch_n),
                          "time_share": ch_ms / ms},
             "kernels_us": {k: round(1e3 * v[1] / max(1, v[0]), 2) for k, v in kt.items()},
+            "attention_roofline": attn_roof,
             "clocks": clocks.summary(local),
         }
         if sweep:

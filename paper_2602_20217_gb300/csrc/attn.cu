@@ -605,6 +605,26 @@ __global__ void __launch_bounds__(128) attn_merge_kernel(const AttnArgs a) {
     const int nch = attn_chunk_of(pos) + 1;
     constexpr int S = HD + kPartPad;
     const float* base = a.part + ((size_t)r * a.hq + hq_idx) * a.n_chunks_max * S;
+    constexpr int PER = HD / 32;   // dims per lane
+    constexpr int PF = 8;          // this warp's first chunks: o loaded while the maxima are reduced
+    float pre[PF][PER];
+#pragma unroll
+    for (int k = 0; k < PF; ++k) {
+        const int c = warp + kAttnWarps * k;
+        const float* src = base + (size_t)c * S + kPartPad + PER * lane;
+        if (c < nch) {
+            if constexpr (PER == 4) {
+                const float4 v = *reinterpret_cast<const float4*>(src);
+                pre[k][0] = v.x;
+                pre[k][1] = v.y;
+                pre[k][2] = v.z;
+                pre[k][3] = v.w;
+            } else {
+#pragma unroll
+                for (int i = 0; i < PER; ++i) pre[k][i] = src[i];
+            }
+        }
+    }
     float mx = -INFINITY;
     for (int c = tid; c < nch; c += blockDim.x) mx = fmaxf(mx, base[(size_t)c * S]);
     mx = warp_max(mx);
@@ -619,12 +639,20 @@ __global__ void __launch_bounds__(128) attn_merge_kernel(const AttnArgs a) {
         ls = fmaf(w, base[(size_t)c * S + 1], ls);
     }
     const float L = block_sum<kAttnWarps>(ls, red);  // ends with a barrier: wsh is visible
-    constexpr int PER = HD / 32;                     // dims per lane
     float o[PER];
 #pragma unroll
     for (int i = 0; i < PER; ++i) o[i] = 0.f;
+#pragma unroll
+    for (int k = 0; k < PF; ++k) {
+        const int c = warp + kAttnWarps * k;
+        if (c < nch) {
+            const float w = wsh[c];
+#pragma unroll
+            for (int i = 0; i < PER; ++i) o[i] = fmaf(w, pre[k][i], o[i]);
+        }
+    }
 #pragma unroll 8
-    for (int c = warp; c < nch; c += kAttnWarps) {   // unrolled: several chunks' loads in flight
+    for (int c = warp + kAttnWarps * PF; c < nch; c += kAttnWarps) {   // unrolled: several loads in flight
         const float w = wsh[c];
         const float* src = base + (size_t)c * S + kPartPad + PER * lane;
         if constexpr (PER == 4) {
