@@ -184,10 +184,18 @@ def test_tiny_lossless_and_knapsack_policy(tiny):
 
 
 # ------------------------------------------------------------- small bf16
-@pytest.mark.parametrize("hd,qk_norm", [(128, False), (128, True), (64, True), ("wide", True)])
+def g8_bf16(L=2):
+    """Eight query heads per KV head (the Qwen3-32B grouping): a verify pass
+    of R = 5 has 40 query rows per KV head, two rounds of query tiles."""
+    from paper_2602_20217_gb300.configs import ModelShape
+    return ModelShape("g8-bf16", L, 512, 16, 2, 128, 1368, 2000, qk_norm=True, dtype="bf16",
+                      rope_theta=1000000.0)
+
+
+@pytest.mark.parametrize("hd,qk_norm", [(128, False), (128, True), (64, True), ("wide", True), ("g8", True)])
 def test_bf16_logits_tokens_and_lossless(hd, qk_norm):
     from paper_2602_20217_gb300 import synth
-    shape = wide_bf16() if hd == "wide" else small_bf16(hd, qk_norm)
+    shape = wide_bf16() if hd == "wide" else g8_bf16() if hd == "g8" else small_bf16(hd, qk_norm)
     prompt = synth.prompt_tokens(shape, 300, seed=1)
     cfg, w = oracle_model(shape, seed=0)
     m = make(shape, 512)

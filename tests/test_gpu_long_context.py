@@ -32,7 +32,12 @@ def _gpu():
 
 
 def _shape(hd):
+    """hd 128 or 64 with four query heads per KV head; "g8": eight (two rounds
+    of query tiles at R = 5)."""
     from paper_2602_20217_gb300.configs import ModelShape
+    if hd == "g8":
+        return ModelShape("g8-bf16", 2, 512, 16, 2, 128, 1368, 2000, qk_norm=True, dtype="bf16",
+                          rope_theta=1000000.0)
     return ModelShape(f"small-bf16-hd{hd}", 2, 512, 8, 2, hd, 1368, 2000, qk_norm=True, dtype="bf16",
                       rope_theta=500000.0)
 
@@ -78,7 +83,7 @@ def _check_last_greedy_row(m, shape, cfg, w, token, next_token):
     assert token_ok(next_token, ref, 0.05 * np.max(np.abs(ref)))
 
 
-@pytest.mark.parametrize("hd", [128, 64])
+@pytest.mark.parametrize("hd", [128, 64, "g8"])
 def test_attention_sublayer_at_40k_context(hd):
     from paper_2602_20217_gb300 import synth
     from paper_2602_20217_gb300.model import Model
