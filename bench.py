@@ -19,6 +19,7 @@ import json
 import os
 import subprocess
 import sys
+import tempfile
 import time
 
 import numpy as np
@@ -284,8 +285,8 @@ def gpu_arm(args):
     torch.cuda.synchronize()
     ev0 = torch.cuda.Event(enable_timing=True)
     ev1 = torch.cuda.Event(enable_timing=True)
-    clk_path = (os.path.join(ROOT, "gpurun_out", f"clocks_rank{rank}.csv")
-                if os.path.isdir(os.path.join(ROOT, "gpurun_out")) else f"/tmp/ks_clocks_{rank}.csv")
+    clk_dir = args.clocks_dir or tempfile.gettempdir()   # the raw nvidia-smi samples
+    clk_path = os.path.join(clk_dir, f"ks_clocks_rank{rank}.csv")
     clocks = ClockSampler(clk_path)
     with clocks:
         torch.cuda.nvtx.range_push("timed")  # lets a profiler capture exactly these steps
@@ -484,6 +485,8 @@ def main():
                     help="dynamic drafting exit threshold (Sec. 3.5); 0 drafts gamma tokens every step")
     ap.add_argument("--tpt-max-gamma", dest="tpt_max_gamma", type=int, default=7,
                     help="D of Alg. 2 (1..15); the default keeps verify passes at 8 rows or fewer")
+    ap.add_argument("--clocks-dir", dest="clocks_dir", default="",
+                    help="directory for the raw clock samples of the timed region (default: the temp dir)")
     ap.add_argument("--sweep", action="store_true",
                     help="also time jobs over a grid of knapsack budgets and draft lengths")
     ap.add_argument("--sweep-budgets", dest="sweep_budgets", default="0.4,0.5,0.6,0.7,0.8")
