@@ -1,11 +1,12 @@
 """GPU parity at full size: the Llama-3-8B-shaped decoder of the 4096-token
-workload in the launch configuration the bench times (32 layers, bf16,
+workload and the Qwen3-8B-shaped decoder (per-head QK-RMSNorm) of the
+32768-token workload, in the launch configuration the bench times (bf16,
 gamma 4, knapsack mask re-solved every step), against the oracle on sampled
 outputs it can compute one by one.
 
 * Lossless (Sec. 2.1): speculative output equals greedy output bit for bit.
 * LM head (final RMSNorm + lm_head): the GPU's logits of the prefill's last
-  rows (those in the history ring) on 2004 sampled vocabulary rows, from the
+  rows (those in the history ring) on every 64th vocabulary row, from the
   GPU's final states X^(2L).
 * Sublayers f^(i) of the first and last layers (Attn: RMSNorm, QKV, RoPE,
   causal GQA over the GPU's K/V cache, W_o, residual; MLP: RMSNorm, SwiGLU,
@@ -67,11 +68,12 @@ def _check_rows(m, cfg, lw, layer, hist, p, tol=2e-2):
     return max(worst, err)
 
 
-def test_llama8b_4k_bench_configuration():
+@pytest.mark.parametrize("workload", ["llama8b-4k", "qwen8b-32k"])
+def test_bench_configuration(workload):
     from paper_2602_20217_gb300 import knapspec as ks, synth
     from paper_2602_20217_gb300.configs import WORKLOADS
     from paper_2602_20217_gb300.model import Model
-    wl = WORKLOADS["llama8b-4k"]
+    wl = WORKLOADS[workload]
     shape = wl.shape
     cfg = D.OracleConfig.like(shape)
     prompt = synth.prompt_tokens(shape, wl.prompt_len, seed=wl.prompt_seed)
@@ -85,7 +87,7 @@ def test_llama8b_4k_bench_configuration():
     assert p == wl.prompt_len and 1 <= r <= 16
     vocab_rows = np.arange(0, shape.vocab, 64)
     lm = synth.np_weight_rows(shape, wl.weight_seed, 0, "lm_head", vocab_rows).astype(np.float64)
-    h = D.rms_norm(hist[-1], np.ones(shape.d_model), cfg.rms_eps)
+    h = D.rms_norm(hist[-1], np.ones(shape.d_model), cfg.rms_eps)   # final-norm gain: ones
     assert rel_err(m.logits(16)[16 - r:, vocab_rows], h @ lm.T) < 2e-2
     layers = {l: _host_layer(shape, wl.weight_seed, l) for l in (0, shape.n_layers - 1)}
     for l, lw in layers.items():
