@@ -32,7 +32,7 @@ from paper_2602_20217_gb300.configs import WORKLOADS  # noqa: E402
 
 METRIC = "accepted tokens/sec at batch 1 on 1xGB300; decode-step HBM GB/s vs ~8 TB/s peak"
 UNIT = "tokens/s"
-DEFAULT_WORKLOAD = "llama8b-4k"
+DEFAULT_WORKLOAD = "qwen32b-64k"   # the largest configuration that fits one GPU
 
 
 def chain_traffic(bytes_per_launch: float):
@@ -112,6 +112,24 @@ def progress(msg: str):
     print(f"[bench {time.time() - _T0:7.1f}s] {msg}", file=sys.stderr, flush=True)
 
 
+def cpu_model() -> str:
+    """The host CPU's model name (lscpu, else /proc/cpuinfo)."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.startswith("Model name:"):
+                return line.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    try:
+        for line in open("/proc/cpuinfo"):
+            if line.lower().startswith(("model name", "cpu model")):
+                return line.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    return "unknown"
+
+
 def cpu_baseline(workload: str, steps: int = 1, warmup: int = 0, timeout: float = 300.0) -> dict:
     cores = os.cpu_count() or 1
     env = dict(os.environ)
@@ -125,7 +143,7 @@ def cpu_baseline(workload: str, steps: int = 1, warmup: int = 0, timeout: float 
         raise RuntimeError("oracle baseline failed: " + out.stderr[-2000:])
     t_token = float(out.stdout.strip().splitlines()[-1])
     sh = WORKLOADS[workload].shape
-    return {"value": 1.0 / t_token, "unit": UNIT, "cores": cores, "kind": "oracle",
+    return {"value": 1.0 / t_token, "unit": UNIT, "cores": cores, "cpu_model": cpu_model(), "kind": "oracle",
             "sample": (f"fp64 numpy oracle, greedy decode token at {WORKLOADS[workload].prompt_len} context: "
                        f"layer 0 Attn+MLP (synthetic KV) x {sh.n_layers} layers + 1/32 of LM-head rows x 32; "
                        f"{steps} timed repeats; every emitted token counts as accepted")}
@@ -221,7 +239,7 @@ def gpu_arm(args):
     gamma = args.gamma or wl.gammas[len(wl.gammas) // 2]
     prompt = synth.prompt_tokens(sh, wl.prompt_len, seed=wl.prompt_seed)
     g_max = max(gamma, int(args.tpt_max_gamma)) if args.policy == "tpt" or args.sweep else gamma
-    max_seq = wl.prompt_len + (max(args.steps, args.warmup) + 2) * (g_max + 1) + args.e2e_tokens + 64
+    max_seq = wl.prompt_len + (max(args.steps, args.warmup) + 2) * (g_max + 1) + (args.e2e_tokens or wl.new_tokens) + 64
     t0 = time.time()
     model = Model(sh, max_seq=max_seq, seed=wl.weight_seed)
     torch.cuda.synchronize()
@@ -276,9 +294,10 @@ def gpu_arm(args):
     progress("warm-up")
     rewind()
     ks.ks_generate_speculative(h, params(args.warmup), 1 << 30)
-    # timed region: exactly K speculation steps, device time on the model's stream
+    # timed region: exactly K speculation steps, device time on the model's
+    # stream, no instrumentation (kernels overlap through programmatic
+    # dependent launch as in normal use)
     rewind()
-    ks.ks_kernel_timing(h, ks.KLASS["chain"], True)
     launches0 = ks.ks_launch_count(h)
     if dist:
         dist.barrier()
@@ -299,29 +318,56 @@ def gpu_arm(args):
         dist.barrier()
     ms = ev0.elapsed_time(ev1)
     launches = ks.ks_launch_count(h) - launches0
+    tokens = int(st.steps + st.accepted)
+
+    # the same K steps again with CUDA events around every chain-kernel
+    # launch: its per-launch duration for the roofline object (the events
+    # serialise the launches, so this pass is slower than the timed one)
+    progress("instrumented pass of the same steps")
+    rewind()
+    ks.ks_kernel_timing(h, ks.KLASS["chain"], True)
+    i0 = torch.cuda.Event(enable_timing=True)
+    i1 = torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    i0.record(stream)
+    _, st_i, _ = ks.ks_generate_speculative(h, params(args.steps), 1 << 30)
+    i1.record(stream)
+    torch.cuda.synchronize()
+    ms_instr = i0.elapsed_time(i1)
     ch_n, ch_ms = ks.ks_kernel_time(h, ks.KLASS["chain"])
     ch_bytes = ks.ks_kernel_bytes(h, ks.KLASS["chain"])
     ks.ks_kernel_timing(h, ks.KLASS["chain"], False)
-    tokens = int(st.steps + st.accepted)
+    assert int(st_i.steps + st_i.accepted) == tokens, "the instrumented pass decoded differently"
 
+    e2e_tokens = args.e2e_tokens or wl.new_tokens
     # e2e: the public call with host output buffers, wall clock, for a
     # generation job of e2e_tokens tokens (the prompt already prefilled)
     rewind()
     h2d0, d2h0 = ks.ks_transfer_bytes(h)
     t0 = time.perf_counter()
-    progress("timed region done; end-to-end job")
-    out, est, eacc = ks.ks_generate_speculative(h, params(0), args.e2e_tokens)
+    progress("end-to-end job")
+    out, est, eacc = ks.ks_generate_speculative(h, params(0), e2e_tokens)
     e2e_s = time.perf_counter() - t0
     h2d1, d2h1 = ks.ks_transfer_bytes(h)
     e2e_tok = int(est.steps + est.accepted)
-    # the same library's plain greedy decode of the same job
+    # the same library's plain greedy decode of the same job, wall clock
     rewind()
     t0 = time.perf_counter()
     progress("greedy job")
-    ar = ks.ks_decode_greedy(h, args.e2e_tokens)
-    progress("greedy job done")
+    ar = ks.ks_decode_greedy(h, e2e_tokens)
     ar_s = time.perf_counter() - t0
     lossless = bool(np.array_equal(out, ar))
+    # and on the device clock, next to `value`
+    rewind()
+    g0 = torch.cuda.Event(enable_timing=True)
+    g1 = torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    g0.record(stream)
+    ks.ks_decode_greedy(h, e2e_tokens)
+    g1.record(stream)
+    torch.cuda.synchronize()
+    ar_dev = (e2e_tokens - 1) / (g0.elapsed_time(g1) * 1e-3)
+    progress("greedy job done")
 
     sweep = []
     if args.sweep:
@@ -336,34 +382,34 @@ def gpu_arm(args):
             e1.record(stream)
             torch.cuda.synchronize()
             return r, e0.elapsed_time(e1) * 1e-3
-        _, t_ar = timed(lambda: ks.ks_decode_greedy(h, args.e2e_tokens))
-        sweep.append({"policy": "greedy", "tokens_per_s": (args.e2e_tokens - 1) / t_ar})
+        _, t_ar = timed(lambda: ks.ks_decode_greedy(h, e2e_tokens))
+        sweep.append({"policy": "greedy", "tokens_per_s": (e2e_tokens - 1) / t_ar})
         for g in sorted({int(x) for x in args.sweep_gammas.split(",")}):
             for bf in [float(x) for x in args.sweep_budgets.split(",")]:
                 p = ks.KsSpecParams(g, 1, None, lat, bf, int(args.resolve_every), 0)
-                (o, sst, _a), t = timed(lambda: ks.ks_generate_speculative(h, p, args.e2e_tokens))
+                (o, sst, _a), t = timed(lambda: ks.ks_generate_speculative(h, p, e2e_tokens))
                 n_tok = int(sst.steps + sst.accepted)
                 sweep.append({"gamma": g, "budget_frac": bf, "tokens_per_s": n_tok / t,
-                              "vs_greedy": (n_tok / t) / ((args.e2e_tokens - 1) / t_ar),
+                              "vs_greedy": (n_tok / t) / ((e2e_tokens - 1) / t_ar),
                               "alpha": float(sst.accepted) / max(1, sst.drafted),
                               "tokens_per_step": n_tok / max(1, sst.steps),
                               "skipped_attn_mlp": [int(sst.attn_skipped), int(sst.mlp_skipped)]})
         # the TPT stage (Alg. 2) picks the layer set and gamma itself
         p = ks.KsSpecParams(gamma, 2, None, lat, 0.0, int(args.tpt_every), 0, int(args.tpt_candidates), tpt_d)
-        (o, sst, _a), t = timed(lambda: ks.ks_generate_speculative(h, p, args.e2e_tokens))
+        (o, sst, _a), t = timed(lambda: ks.ks_generate_speculative(h, p, e2e_tokens))
         n_tok = int(sst.steps + sst.accepted)
         sweep.append({"policy": f"tpt every {args.tpt_every} steps, K {args.tpt_candidates}, D {tpt_d}",
-                      "tokens_per_s": n_tok / t, "vs_greedy": (n_tok / t) / ((args.e2e_tokens - 1) / t_ar),
+                      "tokens_per_s": n_tok / t, "vs_greedy": (n_tok / t) / ((e2e_tokens - 1) / t_ar),
                       "alpha": float(sst.accepted) / max(1, sst.drafted),
                       "mean_gamma": float(sst.drafted) / max(1, sst.steps),
                       "tokens_per_step": n_tok / max(1, sst.steps),
                       "skipped_attn_mlp": [int(sst.attn_skipped), int(sst.mlp_skipped)]})
         # the dynamic drafting exit of Sec. 3.5 (tau_conf 0.7) on the default knapsack policy
         p = ks.KsSpecParams(gamma, 1, None, lat, float(args.budget_frac), int(args.resolve_every), 0, 0, 0, 0.7)
-        (o, sst, _a), t = timed(lambda: ks.ks_generate_speculative(h, p, args.e2e_tokens))
+        (o, sst, _a), t = timed(lambda: ks.ks_generate_speculative(h, p, e2e_tokens))
         n_tok = int(sst.steps + sst.accepted)
         sweep.append({"policy": f"knapsack, gamma {gamma} max, budget {args.budget_frac}, dynamic exit tau_conf 0.7",
-                      "tokens_per_s": n_tok / t, "vs_greedy": (n_tok / t) / ((args.e2e_tokens - 1) / t_ar),
+                      "tokens_per_s": n_tok / t, "vs_greedy": (n_tok / t) / ((e2e_tokens - 1) / t_ar),
                       "alpha": float(sst.accepted) / max(1, sst.drafted),
                       "drafts_per_step": float(sst.drafted) / max(1, sst.steps),
                       "tokens_per_step": n_tok / max(1, sst.steps)})
@@ -379,21 +425,21 @@ def gpu_arm(args):
         dp_s = time.perf_counter() - t0
         dm = np.ascontiguousarray(dmask, np.uint8)
         p = ks.KsSpecParams(int(dgamma), 0, dm.ctypes.data_as(ks.C.POINTER(ks.C.c_uint8)), lat, 0.0, 1, 0)
-        (o, sst, _a), t = timed(lambda: ks.ks_generate_speculative(h, p, args.e2e_tokens))
+        (o, sst, _a), t = timed(lambda: ks.ks_generate_speculative(h, p, e2e_tokens))
         n_tok = int(sst.steps + sst.accepted)
         sweep.append({"policy": f"hidden-state DP (Alg. 1, tau 0.5) + TPT grid (D {tpt_d}), selected once",
                       "dp_seconds": dp_s, "dp_candidates": int(len(djs)), "gamma": int(dgamma),
                       "skipped_attn_mlp": [int(np.sum(dmask[0::2] == 0)), int(np.sum(dmask[1::2] == 0))],
-                      "tokens_per_s": n_tok / t, "vs_greedy": (n_tok / t) / ((args.e2e_tokens - 1) / t_ar),
+                      "tokens_per_s": n_tok / t, "vs_greedy": (n_tok / t) / ((e2e_tokens - 1) / t_ar),
                       "alpha": float(sst.accepted) / max(1, sst.drafted),
                       "tokens_per_step": n_tok / max(1, sst.steps)})
         # sampling mode (Sec. 2.1; nucleus sampling with T 0.7, top-k 50, top-p 0.95 as in Sec. 4)
         p = ks.KsSpecParams(gamma, 1, None, lat, float(args.budget_frac), int(args.resolve_every), 0, 0, 0, 0.0,
                             ks.sampling(0.7, 50, 0.95, 12345))
-        (o, sst, _a), t = timed(lambda: ks.ks_generate_speculative(h, p, args.e2e_tokens))
+        (o, sst, _a), t = timed(lambda: ks.ks_generate_speculative(h, p, e2e_tokens))
         n_tok = int(sst.steps + sst.accepted)
         sweep.append({"policy": f"knapsack, gamma {gamma}, budget {args.budget_frac}, sampling T 0.7 top-k 50 top-p 0.95",
-                      "tokens_per_s": n_tok / t, "vs_greedy": (n_tok / t) / ((args.e2e_tokens - 1) / t_ar),
+                      "tokens_per_s": n_tok / t, "vs_greedy": (n_tok / t) / ((e2e_tokens - 1) / t_ar),
                       "alpha": float(sst.accepted) / max(1, sst.drafted),
                       "tokens_per_step": n_tok / max(1, sst.steps)})
 
@@ -426,14 +472,17 @@ def gpu_arm(args):
                                  (f"TPT stage every {args.tpt_every} step(s), K {args.tpt_candidates}, "
                                   f"D {tpt_d}"))
                                  + (f", dynamic exit tau_conf {args.tau_conf}" if args.tau_conf > 0 else ""),
-                       "l2": "inputs larger than L2 (each step streams the weights, 16+ GB)",
+                       "l2": (f"inputs larger than L2 (each step streams "
+                              f"{(sh.n_layers * (sh.attn_weight_bytes() + sh.mlp_weight_bytes()) + sh.lm_head_bytes()) / 1e9:.1f} GB of weights)"),
                        "parallelism": f"replicas x{world}"},
             "tokens": tokens, "mean_tokens_per_step": tokens / max(1, st.steps),
             "alpha": float(st.accepted) / max(1, st.drafted),
             "mean_gamma": float(st.drafted) / max(1, st.steps),
             "mask_skipped": {"attn": int(st.attn_skipped), "mlp": int(st.mlp_skipped)},
-            "ar_tokens_per_s": (args.e2e_tokens - 1) / ar_s,
-            "spec_vs_ar_e2e": (e2e_tok / e2e_s) / ((args.e2e_tokens - 1) / ar_s),
+            "ar_tokens_per_s": (e2e_tokens - 1) / ar_s,
+            "spec_vs_ar_e2e": (e2e_tok / e2e_s) / ((e2e_tokens - 1) / ar_s),
+            "ar_tokens_per_s_device": ar_dev,
+            "spec_vs_ar_device": (tok_all / (ms_max * 1e-3)) / ar_dev,
             "lossless_vs_ar": lossless,
             "latency_model_ms": {"c1": c1, "c2": c2, "c3": c3},
             "prefill_s": t_prefill, "setup_s": t_setup,
@@ -443,10 +492,11 @@ def gpu_arm(args):
             "gpu_launches": launches,
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak,
-                         "traffic": chain_traffic(ch_bytes / max(1, ch_n)) if wl.name == "llama8b-4k" else None,
+                         "traffic": chain_traffic(ch_bytes / max(1, ch_n)),
                          "kernel": "chain_kernel (chained projections)", "peak_source": peak_kind,
                          "launches_timed": ch_n, "bytes_per_launch": ch_bytes / max(1, ch_n),
-                         "time_share": ch_ms / ms},
+                         "timing": "CUDA events around each launch, in a second pass of the same steps",
+                         "time_share": ch_ms / ms_instr, "instrumented_ms_per_step": ms_instr / args.steps},
             "kernels_us": {k: round(1e3 * v[1] / max(1, v[0]), 2) for k, v in kt.items()},
             "attention_roofline": attn_roof,
             "clocks": clocks.summary(local),
@@ -475,7 +525,8 @@ def main():
     ap.add_argument("--gamma", type=int, default=0)
     ap.add_argument("--budget-frac", dest="budget_frac", type=float, default=0.8)
     ap.add_argument("--resolve-every", dest="resolve_every", type=int, default=1)
-    ap.add_argument("--e2e-tokens", dest="e2e_tokens", type=int, default=256)
+    ap.add_argument("--e2e-tokens", dest="e2e_tokens", type=int, default=0,
+                    help="tokens of the end-to-end and greedy jobs (default: the workload's generation length)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--policy", default="knapsack", choices=["knapsack", "tpt"],
                     help="mask policy of the timed steps: knapsack at --budget-frac, or the TPT stage")

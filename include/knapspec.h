@@ -106,7 +106,10 @@ typedef struct {
  * kind 0: App. C model t_MLP = c1, t_Attn(n) = c2 n + c3, turned into integer
  *         weights by Sec. 3.4: Delta = min(t_Attn(n), t_MLP),
  *         w = round(t / Delta) (half away from zero, at least 1).
- * kind 1: explicit integer units per sublayer, units[2L] (host), all >= 1. */
+ *         Requires c1 > 0, c2 >= 0, c3 >= 0 (finite), t_Attn(n) > 0 at the
+ *         context length used, and max(t_Attn, t_MLP) / min(t_Attn, t_MLP)
+ *         <= 65535; otherwise the call taking it returns KS_ERR_INVALID_ARG.
+ * kind 1: explicit integer units per sublayer, units[2L] (host), 1..65535. */
 typedef struct {
     int32_t kind;
     double c1, c2, c3;
@@ -275,9 +278,12 @@ ks_status ks_select_mask(const ks_latency* lat, const float* sims, int64_t conte
  * arguments; budget_units must be 0..KS_SELECT_STATIC_MAX_BUDGET (larger
  * budgets return KS_ERR_INVALID_ARG).  The call allocates nothing: no
  * cudaMalloc, cudaFree or allocating library routine.
- * The first call on a device looks up the array's device address
- * (cudaGetSymbolAddress) with that device current; make that first call
- * before any stream capture.  All calls share the one array and the kernel
+ * Every call looks up the array's device address (cudaGetSymbolAddress)
+ * on the current device, so a context created after cudaDeviceReset gets its
+ * own copy.  With CUDA's lazy module loading, the first call on a device may
+ * load this library's device code, and the driver then reserves memory for
+ * the module and this array; make that first call during start-up, before
+ * any stream capture.  All calls share the one array and the kernel
  * rewrites every table entry it reads, so no state leaks from one call to
  * the next; two calls whose kernels overlap on the GPU (different streams)
  * race on the array and must be ordered by the caller. */

@@ -32,8 +32,10 @@
 //    the same argmax); the CTA whose count completes the phase reads it.
 //    Partials are double buffered, so consumers never wait for an epilogue.
 // A stage is full when both loaders have arrived and all bytes have landed.
-// Deadlock-free without co-residency: items are only claimed by running
-// CTAs, a CTA works its claims in order, and the lowest unfinished phase
+// A CTA's first unit of each phase is fixed by its index; further units are
+// claimed from per-phase atomic queues.  Deadlock-free: every CTA of the grid
+// becomes resident once the kernels before it finish (the grid is sized to
+// fit), a CTA works its units in phase order, and the lowest unfinished phase
 // always has all its inputs.  Every wait is bounded (2 s): on expiry the
 // status word is set and the CTA leaves.
 #include "common.cuh"
@@ -350,23 +352,32 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
                 ++t;
                 return true;
             };
-            // Items are claimed from the start: this launch's queues were
-            // zeroed by the launch before the previous one (counter sets
-            // alternate), which has completed.  Weight boxes need no input,
-            // so the first S stages go out while the previous kernel runs.
+            // Work assignment per phase: the CTA's first unit is fixed by its
+            // index (unit blockIdx.x, if the phase has that many), so phases
+            // with about one unit per CTA (W_o, W_down, QKV) spread over every
+            // CTA; further units come from the phase's atomic queue, offset by
+            // the grid size.  This launch's queues were zeroed by the launch
+            // before the previous one (counter sets alternate), which has
+            // completed.  Weight boxes need no input, so the first S stages
+            // go out while the previous kernel runs.  No deadlock: every CTA
+            // of the grid is co-resident once the kernels before it finish,
+            // and a CTA finishes its units of a phase before it waits for the
+            // next phase's inputs.
+            const int grid = (int)gridDim.x;
             int k = 0;
             Phase P = decode(a, 0);
-            int it = atomicAdd(&queue[0], 1);
+            int it = (int)blockIdx.x;
             while (ok) {   // `it` counts units: item it / n_sl, K-slice it % n_sl
                 if (it >= P.n_units) {
                     if (++k >= a.n_phases) break;
                     P = decode(a, k);
-                    it = atomicAdd(&queue[k], 1);
+                    it = (int)blockIdx.x;
                     continue;
                 }
-                const int next = atomicAdd(&queue[k], 1);  // claimed ahead: its latency hides behind the stream
-                // (the ticket is first needed at the unit's last stage, so its
+                // claimed ahead: its latency hides behind the stream (the
+                // ticket is first needed at the unit's last stage, so its
                 // round trip overlaps the unit's other stages)
+                const int next = P.n_units > grid ? grid + atomicAdd(&queue[k], 1) : INT_MAX;
                 const int item = it / P.n_sl, sl = it - item * P.n_sl;
                 const int kt0 = sl * P.sl_len, kt1 = min(P.tpi, kt0 + P.sl_len);
                 for (int kt = kt0; kt < kt1 && ok; ++kt)

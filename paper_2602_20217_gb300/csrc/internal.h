@@ -149,6 +149,12 @@ cudaError_t launch_cosine(const void* X, const void* Y, int dtype, int64_t n_pai
                           int d, int64_t pair_stride, const int32_t* row_index, float* out,
                           cudaStream_t s);
 
+// Latency model checks shared by every entry point that takes one: kind 0
+// needs c1 > 0, c2, c3 >= 0, t_Attn(context_len) = c2 n + c3 > 0 and the
+// larger of t_Attn, t_MLP at most 65535 times the smaller; kind 1 needs
+// units in 1..65535.
+bool latency_valid(const ks_latency* lat, int32_t n_sublayers, int64_t context_len);
+
 // Last error text for ks_last_error (thread-local).
 void set_error(const char* fmt, ...);
 

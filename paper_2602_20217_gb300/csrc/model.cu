@@ -1414,13 +1414,8 @@ ks_status ks_history_similarities(ks_model* m, float* sims, int32_t* rows_used) 
     return KS_OK;
 }
 
-static bool latency_ok(const ks_latency& lat, int nsub) {
-    bool ok = lat.kind == 0 ? (lat.c1 > 0 && lat.c2 >= 0 && lat.c3 >= 0 && std::isfinite(lat.c1) &&
-                               std::isfinite(lat.c2) && std::isfinite(lat.c3))
-                            : (lat.kind == 1 && lat.units);
-    if (ok && lat.kind == 1)
-        for (int i = 0; i < nsub; ++i) ok = ok && lat.units[i] >= 1 && lat.units[i] <= 65535;
-    return ok;
+static bool latency_ok(const ks_latency& lat, int nsub, int64_t context_len) {
+    return latency_valid(&lat, nsub, context_len);
 }
 
 ks_status ks_select_tpt(ks_model* m, const ks_latency* lat, int32_t n_candidates, int32_t max_gamma,
@@ -1431,7 +1426,7 @@ ks_status ks_select_tpt(ks_model* m, const ks_latency* lat, int32_t n_candidates
         return KS_ERR_INVALID_ARG;
     }
     if (n_candidates < 1 || n_candidates > KS_TPT_MAX_CANDIDATES || max_gamma < 1 ||
-        max_gamma >= m->cfg.max_rows || !latency_ok(*lat, m->nsub)) {
+        max_gamma >= m->cfg.max_rows || !latency_ok(*lat, m->nsub, m->p)) {
         set_error("ks_select_tpt: bad argument");
         return KS_ERR_INVALID_ARG;
     }
@@ -1542,7 +1537,7 @@ ks_status ks_select_dp(ks_model* m, const ks_latency* lat, float tau, int32_t ma
     const ks_config& c = m->cfg;
     const int nsub = m->nsub, d = c.d_model, L = c.n_layers;
     if (max_gamma < 1 || max_gamma >= c.max_rows || max_states < 1 || max_states > kDpMaxStates || max_rows < 1 ||
-        !std::isfinite(tau) || !latency_ok(*lat, nsub)) {
+        !std::isfinite(tau) || !latency_ok(*lat, nsub, m->p)) {
         set_error("ks_select_dp: bad argument");
         return KS_ERR_INVALID_ARG;
     }
@@ -1743,7 +1738,7 @@ ks_status ks_generate_speculative(ks_model* m, const ks_spec_params* prm, int32_
                   "and no dynamic exit");
         return KS_ERR_INVALID_ARG;
     }
-    if (prm->policy != 0 && !latency_ok(prm->latency, nsub)) {
+    if (prm->policy != 0 && !latency_ok(prm->latency, nsub, m->p)) {
         set_error("ks_generate_speculative: bad latency model");
         return KS_ERR_INVALID_ARG;
     }
@@ -1755,6 +1750,10 @@ ks_status ks_generate_speculative(ks_model* m, const ks_spec_params* prm, int32_
     std::vector<int32_t> toks(m->cfg.max_rows + 1);
     int gamma = prm->gamma;
     while (n < n_tokens && (prm->max_steps <= 0 || st.steps < prm->max_steps)) {
+        if (prm->policy != 0 && st.steps % prm->resolve_every == 0 && !latency_ok(prm->latency, nsub, m->p)) {
+            set_error("ks_generate_speculative: latency model invalid at context %d", m->p);
+            return KS_ERR_INVALID_ARG;
+        }
         if (prm->policy == 2 && st.steps % prm->resolve_every == 0) {
             // TPT stage: the next mask and draft length
             KS_TRY(tpt_stage(m, &prm->latency, prm->tpt_candidates, prm->tpt_max_gamma, nullptr));

@@ -15,7 +15,6 @@
 #include "internal.h"
 
 #include <cmath>
-#include <mutex>
 
 namespace ks {
 
@@ -324,22 +323,33 @@ cudaError_t launch_tpt(const ks_latency* lat, int64_t n, int n_items, int n_laye
     return cudaGetLastError();
 }
 
-static ks_status check_latency(const ks_latency* lat, int32_t n) {
-    if (!lat) return KS_ERR_INVALID_ARG;
+}  // namespace ks
+
+// Sec. 3.4 / App. C: the integer weights are round(t / Delta) with Delta =
+// min(t_Attn(n), t_MLP), t_Attn(n) = c2 n + c3, t_MLP = c1.  Both times must
+// be positive, and the larger may be at most 65535 times the smaller (the
+// limit of explicit units), or the quotient would not be a valid weight.
+bool ks::latency_valid(const ks_latency* lat, int32_t n_sublayers, int64_t context_len) {
+    if (!lat) return false;
     if (lat->kind == 0) {
         if (!(lat->c1 > 0.0) || !(lat->c2 >= 0.0) || !(lat->c3 >= 0.0) || !std::isfinite(lat->c1) ||
-            !std::isfinite(lat->c2) || !std::isfinite(lat->c3))
-            return KS_ERR_INVALID_ARG;
-        return KS_OK;
+            !std::isfinite(lat->c2) || !std::isfinite(lat->c3) || context_len < 0)
+            return false;
+        const double ta = lat->c2 * (double)context_len + lat->c3;
+        if (!(ta > 0.0) || !std::isfinite(ta)) return false;
+        const double hi = std::fmax(ta, lat->c1), lo = std::fmin(ta, lat->c1);
+        return hi / lo <= 65535.0;
     }
     if (lat->kind == 1) {
-        if (!lat->units) return KS_ERR_INVALID_ARG;
-        for (int i = 0; i < n; ++i)
-            if (lat->units[i] < 1 || lat->units[i] > 65535) return KS_ERR_INVALID_ARG;
-        return KS_OK;
+        if (!lat->units) return false;
+        for (int i = 0; i < n_sublayers; ++i)
+            if (lat->units[i] < 1 || lat->units[i] > 65535) return false;
+        return true;
     }
-    return KS_ERR_INVALID_ARG;
+    return false;
 }
+
+namespace ks {
 
 // ------------------------------------------------ allocation-free variant
 // Work tables of ks_select_mask_static: one array for the whole process on
@@ -352,24 +362,14 @@ constexpr size_t kStaticScratchBytes =
     256;
 static __device__ __align__(256) unsigned char g_select_scratch[kStaticScratchBytes];
 
-static std::mutex g_static_mu;
-static void* g_static_ptr[128] = {};
-
-// Device address of g_select_scratch on the current device, looked up once
-// per device (the first call on a device does the lookup).
+// Device address of g_select_scratch on the current device.  Looked up on
+// every call (cheap once the module is loaded), so a new primary context
+// after cudaDeviceReset gets the address of its own copy of the array.
 static cudaError_t static_scratch(void** out) {
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_select_scratch);
     if (e != cudaSuccess) return e;
-    if (dev < 0 || dev >= 128) return cudaErrorInvalidDevice;
-    std::lock_guard<std::mutex> lock(g_static_mu);
-    if (g_static_ptr[dev] == nullptr) {
-        void* p = nullptr;
-        e = cudaGetSymbolAddress(&p, g_select_scratch);
-        if (e != cudaSuccess) return e;
-        g_static_ptr[dev] = p;
-    }
-    *out = g_static_ptr[dev];
+    *out = p;
     return cudaSuccess;
 }
 
@@ -394,8 +394,8 @@ extern "C" ks_status ks_select_mask_static(const ks_latency* lat, const float* s
                   budget_units, kStaticCap);
         return KS_ERR_INVALID_ARG;
     }
-    if (check_latency(lat, n_sublayers) != KS_OK) {
-        set_error("ks_select_mask_static: bad latency model");
+    if (!latency_valid(lat, n_sublayers, context_len)) {
+        set_error("ks_select_mask_static: bad latency model (times must be positive, ratio at most 65535)");
         return KS_ERR_INVALID_ARG;
     }
     void* scratch = nullptr;
@@ -453,8 +453,8 @@ extern "C" ks_status ks_select_mask(const ks_latency* lat, const float* sims, in
         set_error("ks_select_mask: bad n_sublayers / budget / context_len");
         return KS_ERR_INVALID_ARG;
     }
-    if (check_latency(lat, n_sublayers) != KS_OK) {
-        set_error("ks_select_mask: bad latency model");
+    if (!latency_valid(lat, n_sublayers, context_len)) {
+        set_error("ks_select_mask: bad latency model (times must be positive, ratio at most 65535)");
         return KS_ERR_INVALID_ARG;
     }
     if ((reinterpret_cast<uintptr_t>(scratch) & 15) != 0) {

@@ -127,15 +127,17 @@ def torch_bits(key: int, start: int, n: int, device):
     return z ^ _t_lsr(z, 31)
 
 
-def torch_normal_(out, key: int, std: float, chunk: int = 1 << 25):
-    """Fill a contiguous fp32/bf16 tensor with the generator's values, in chunks."""
+def torch_normal_(out, key: int, std: float, chunk: int = 1 << 25, start: int = 0):
+    """Fill a contiguous fp32/bf16 tensor with the generator's values for
+    element indices start, start + 1, ... (a slice of a larger tensor's
+    stream when start > 0), in chunks."""
     import torch
     flat = out.view(-1)
     total = flat.numel()
     scale = float(np.float32(std / IH_SD))
     for s in range(0, total, chunk):
         n = min(chunk, total - s)
-        z = torch_bits(key, s, n, out.device)
+        z = torch_bits(key, start + s, n, out.device)
         lanes = (z & 0xFFFF) + (_t_lsr(z, 16) & 0xFFFF) + (_t_lsr(z, 32) & 0xFFFF) + _t_lsr(z, 48)
         v = (lanes - IH_MEAN).to(torch.float32) * scale
         flat[s:s + n].copy_(v.to(flat.dtype))

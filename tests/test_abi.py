@@ -131,6 +131,22 @@ def test_select_mask_argument_checks(lib):
     assert call(bad) == ks.KS_ERR_INVALID_ARG
     bad, _ = ks.latency(5)
     assert call(bad) == ks.KS_ERR_INVALID_ARG
+    # t_Attn(n) = c2 n + c3 must be positive at the context length used
+    zero_attn, _ = ks.latency(0, 0.3, 0.0, 0.0)
+    assert call(zero_attn, ctx=0) == ks.KS_ERR_INVALID_ARG
+    assert call(zero_attn, ctx=4096) == ks.KS_ERR_INVALID_ARG
+    # the ratio of the two times must fit the integer weights (at most 65535)
+    lopsided, _ = ks.latency(0, 1.0, 0.0, 1.0 / 70000.0)
+    assert call(lopsided) == ks.KS_ERR_INVALID_ARG
+    ok_ratio, _ = ks.latency(0, 1.0, 0.0, 1.0 / 60000.0)
+    assert call(ok_ratio, nbytes=16) == ks.KS_ERR_WORKSPACE   # passes the model check, fails the next one
+    growing, _ = ks.latency(0, 1e-9, 1e-9, 0.0)            # t_Attn / t_MLP = n: valid at 4096, not at 1e6
+    assert call(growing, nbytes=16) == ks.KS_ERR_WORKSPACE
+    assert call(growing, ctx=1000000) == ks.KS_ERR_INVALID_ARG
+    # the allocation-free variant applies the same checks before any device work
+    for bad_lat, ctx in [(zero_attn, 0), (lopsided, 4096), (growing, 1000000)]:
+        assert lib.ks_select_mask_static(C.byref(bad_lat), fake, ctx, 8, 5, fake, None, None,
+                                         None) == ks.KS_ERR_INVALID_ARG
     assert args
 
 

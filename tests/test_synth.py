@@ -24,6 +24,10 @@ def test_numpy_and_torch_streams_agree():
     t = torch.empty(4096, dtype=torch.float32)
     synth.torch_normal_(t, key, 0.02, chunk=1000)
     assert np.array_equal(t.numpy(), synth.np_normal32(key, np.arange(4096, dtype=np.uint64), 0.02))
+    # a slice of the stream from an element offset equals the same slice of the whole
+    u = torch.empty(1500, dtype=torch.float32)
+    synth.torch_normal_(u, key, 0.02, chunk=700, start=2000)
+    assert np.array_equal(u.numpy(), t.numpy()[2000:3500])
 
 
 def test_bf16_rounding_matches_torch():
