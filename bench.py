@@ -64,43 +64,52 @@ def peaks():
 
 
 # ------------------------------------------------------------ oracle arm
-def oracle_sample_seconds(workload: str, seed: int = 0) -> dict:
-    """Time the fp64 oracle on a bounded sample of one greedy decode token:
-    layer 0's Attn + MLP sublayers at the workload's context (synthetic KV
-    cache) and 1/32 of the LM head rows; the token time is scaled to all
-    layers and the full vocabulary."""
-    from oracle import decoder as D
-    from paper_2602_20217_gb300 import synth
-    wl = WORKLOADS[workload]
-    sh = wl.shape
-    cfg = D.OracleConfig.like(sh)
-    lw = {k: synth.np_weight(sh, seed, 0, k).astype(np.float64) for k in synth.weight_shapes(sh)["layer"]}
-    n = wl.prompt_len
-    rng_key = synth.stream_key(seed, 0, "kv")
-    kv = synth.np_normal32(rng_key, np.arange(2 * sh.n_kv_heads * (n + 1) * sh.head_dim, dtype=np.uint64), 1.0)
-    kv = kv.astype(np.float64).reshape(2, sh.n_kv_heads, n + 1, sh.head_dim)
-    K, V = kv[0].copy(), kv[1].copy()
-    x = synth.np_weight_rows(sh, seed, 0, "embed", [7]).astype(np.float64)
-    rows = np.arange(0, sh.vocab, 32)
-    W_lm = synth.np_weight_rows(sh, seed, 0, "lm_head", rows).astype(np.float64)
-    gain = np.ones(sh.d_model)
-    t0 = time.perf_counter()
-    x1 = D.attn_sublayer(cfg, lw, x, np.array([n]), K, V)
-    x2 = D.mlp_sublayer(cfg, lw, x1)
-    t1 = time.perf_counter()
-    _ = D.rms_norm(x2, gain, cfg.rms_eps) @ W_lm.T
-    t2 = time.perf_counter()
-    return {"t_layer": t1 - t0, "t_lm_slice": t2 - t1,
-            "t_token": sh.n_layers * (t1 - t0) + (sh.vocab / len(rows)) * (t2 - t1)}
+class OracleSample:
+    """A bounded sample of one greedy decode token of the workload for the
+    plain fp32 C++ oracle (one thread): one layer's Attn + MLP sublayers at
+    the workload's context (a synthetic KV cache) and 1/32 of the LM-head
+    rows; the token time scales them to all layers and the full vocabulary.
+    The sample's weights and cache are seeded normal values of the workload's
+    shapes (the oracle's operation count does not depend on the values)."""
+
+    def __init__(self, workload: str, seed: int = 0):
+        from dataclasses import replace
+        from oracle import cxx
+        from paper_2602_20217_gb300 import synth
+        wl = WORKLOADS[workload]
+        self.sh = sh = wl.shape
+        rng = np.random.default_rng(seed)
+        normal = lambda shape: (0.02 * rng.standard_normal(shape, dtype=np.float32))
+        self.lm_rows = (sh.vocab + 31) // 32
+        sample = replace(sh, n_layers=1, vocab=self.lm_rows, dtype="f32")
+        shapes = synth.weight_shapes(sample)
+        w = {k: (np.ones(v, np.float32) if k in synth.NORM_KINDS else normal(v)) for k, v in shapes["global"].items()}
+        w["layers"] = [{k: (np.ones(v, np.float32) if k in synth.NORM_KINDS else normal(v))
+                        for k, v in shapes["layer"].items()}]
+        self.m = cxx.Model(sample, w)
+        self.n = wl.prompt_len
+        self.K = rng.standard_normal((sh.n_kv_heads, self.n + 1, sh.head_dim), dtype=np.float32)
+        self.V = rng.standard_normal((sh.n_kv_heads, self.n + 1, sh.head_dim), dtype=np.float32)
+        self.x = normal((1, sh.d_model)) * 50.0
+
+    def token_seconds(self) -> float:
+        t0 = time.perf_counter()
+        x1 = self.m.attn_sublayer(0, self.x, [self.n], self.K, self.V)
+        x2 = self.m.mlp_sublayer(0, x1)
+        t1 = time.perf_counter()
+        self.m.final_logits(x2)
+        t2 = time.perf_counter()
+        return self.sh.n_layers * (t1 - t0) + (self.sh.vocab / self.lm_rows) * (t2 - t1)
 
 
 def run_oracle_arm(args, workload):
-    """Runs in a child process with a fixed BLAS thread count; prints JSON."""
+    """Runs in a child process; returns the mean token time over the timed samples."""
+    smp = OracleSample(workload)
     samples = []
     for i in range(args.warmup + args.steps):
-        r = oracle_sample_seconds(workload)
+        t = smp.token_seconds()
         if i >= args.warmup:
-            samples.append(r["t_token"])
+            samples.append(t)
     return float(np.mean(samples))
 
 
@@ -130,23 +139,23 @@ def cpu_model() -> str:
     return "unknown"
 
 
-def cpu_baseline(workload: str, steps: int = 1, warmup: int = 0, timeout: float = 300.0) -> dict:
-    cores = os.cpu_count() or 1
-    env = dict(os.environ)
-    for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
-        env[k] = str(cores)
+def cpu_baseline(workload: str, steps: int = 1, warmup: int = 0, timeout: float = 600.0) -> dict:
+    """The plain fp32 C++ oracle, single-threaded, on a bounded sample (see
+    oracle_sample_seconds), in a child process."""
     code = ("import sys, json; sys.path.insert(0, %r); import bench; "
             "print(json.dumps(bench.run_oracle_arm(type('A', (), {'steps': %d, 'warmup': %d})(), %r)))"
             % (ROOT, steps, warmup, workload))
-    out = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True, timeout=timeout)
+    out = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, timeout=timeout)
     if out.returncode != 0:
         raise RuntimeError("oracle baseline failed: " + out.stderr[-2000:])
     t_token = float(out.stdout.strip().splitlines()[-1])
-    sh = WORKLOADS[workload].shape
-    return {"value": 1.0 / t_token, "unit": UNIT, "cores": cores, "cpu_model": cpu_model(), "kind": "oracle",
-            "sample": (f"fp64 numpy oracle, greedy decode token at {WORKLOADS[workload].prompt_len} context: "
-                       f"layer 0 Attn+MLP (synthetic KV) x {sh.n_layers} layers + 1/32 of LM-head rows x 32; "
-                       f"{steps} timed repeats; every emitted token counts as accepted")}
+    wl = WORKLOADS[workload]
+    sh = wl.shape
+    return {"value": 1.0 / t_token, "unit": UNIT, "cores": 1, "cpu_model": cpu_model(), "kind": "oracle",
+            "sample": (f"plain fp32 C++ oracle (oracle/cpp, one thread), greedy decode token at "
+                       f"{wl.prompt_len} context: one layer's Attn+MLP (synthetic KV cache) x {sh.n_layers} layers "
+                       f"+ 1/32 of the LM-head rows x 32; {steps} timed sample(s) after {warmup} untimed; every "
+                       f"emitted token counts as accepted")}
 
 
 def reference_arm(args):
@@ -157,7 +166,7 @@ def reference_arm(args):
     cb = cpu_baseline(wl, steps=args.steps, warmup=args.warmup)
     line = {"metric": METRIC, "value": cb["value"], "unit": UNIT, "n_gpus": args.gpus, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": 1e3 / cb["value"], "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
             "impl": "reference",
             "config": {"workload": wl, "model": WORKLOADS[wl].shape.name, "prompt": WORKLOADS[wl].prompt_len},
             "cpu_baseline": cb,
@@ -206,6 +215,33 @@ class ClockSampler:
         reasons = sorted({names[i] for r in rows for i in range(4) if len(r) > 5 + i and r[5 + i] == "Active"})
         return {"sm_mhz": float(np.median(sm)) if sm else None, "sm_max_mhz": max(mx) if mx else None,
                 "reasons": reasons, "samples": len(rows)}
+
+
+def attention_ms(shape, n: int, seed: int = 0) -> float:
+    """Per-launch time (ms, CUDA events) of the split-KV attention kernel of a
+    greedy step at context n, on a one-layer model with the workload's
+    attention shape (the kernel's time depends on the heads, head size and
+    context, not on the model's depth)."""
+    from dataclasses import replace
+    import torch
+    from paper_2602_20217_gb300 import knapspec as ks, synth
+    from paper_2602_20217_gb300.configs import truncated
+    from paper_2602_20217_gb300.model import Model
+    sh = replace(truncated(shape, 1), vocab=1024)
+    m = Model(sh, max_seq=n + 32, seed=seed)
+    m.prefill(synth.prompt_tokens(sh, n, seed=1))
+    k = ks.KLASS["attn"]
+    ks.ks_kernel_timing(m.h, k, True)
+    m.decode_greedy(3)
+    ks.ks_kernel_timing(m.h, k, False)
+    ks.ks_kernel_timing(m.h, k, True)
+    m.decode_greedy(9)
+    cnt, ms = ks.ks_kernel_time(m.h, k)
+    ks.ks_kernel_timing(m.h, k, False)
+    m.close()
+    del m
+    torch.cuda.empty_cache()
+    return ms / max(1, cnt)
 
 
 def reduce_over_ranks(ms: float, tokens: float, dist=None, device="cpu"):
@@ -258,8 +294,8 @@ def gpu_arm(args):
 
     # Latency model of App. C measured on this GPU at the prompt's context:
     # c1 = MLP sublayer (gate/up + down), c3 = the Attn sublayer's
-    # context-independent kernels (QKV, merge, O-proj), c2 = attention-kernel
-    # time / context length.
+    # context-independent kernels (QKV, query prep, merge, O-proj), c2 =
+    # attention-kernel time / context length.
     progress("model created; prefill")
     t_prefill = prefill()
     progress("prefill done; latency model")
@@ -277,9 +313,17 @@ def gpu_arm(args):
         ks.ks_kernel_timing(h, k, False)
     per = lambda name: kt[name][1] / max(1, kt[name][0])
     c1 = per("gateup") + per("down")
-    c3 = per("qkv") + per("merge") + per("oproj")
-    c2 = per("attn") / wl.prompt_len
-    lat, _keep = ks.latency(0, c1, c2, c3)
+    fixed = per("qkv") + per("prep") + per("merge") + per("oproj")
+    # App. C's profiling sweep: the attention kernel's time at four context
+    # lengths (a one-layer model with this attention shape, R = 1), fitted
+    # with the fixed Attn-sublayer kernels by least squares (ks_fit_latency)
+    progress("latency sweep")
+    sweep_n = [max(256, wl.prompt_len // 8), max(512, wl.prompt_len // 4), max(1024, wl.prompt_len // 2),
+               wl.prompt_len]
+    sweep_t = [attention_ms(sh, n) for n in sweep_n]
+    lat = ks.ks_fit_latency(sweep_n, [fixed + t for t in sweep_t], [c1])
+    _keep = None
+    c2, c3 = lat.c2, lat.c3
 
     tpt_d = int(args.tpt_max_gamma)   # D of Alg. 2: the longest draft the grid search may pick
 
@@ -433,6 +477,29 @@ def gpu_arm(args):
                       "tokens_per_s": n_tok / t, "vs_greedy": (n_tok / t) / ((e2e_tokens - 1) / t_ar),
                       "alpha": float(sst.accepted) / max(1, sst.drafted),
                       "tokens_per_step": n_tok / max(1, sst.steps)})
+        # Eq. 3's prediction for the DP's best candidates (each at its best
+        # gamma, the fitted latency model at the prompt's context, times in
+        # ms) next to the tokens/s their jobs reach
+        ta, tm = c2 * wl.prompt_len + c3, c1
+
+        def predicted(mask_c, alpha, g):
+            e = sum(alpha ** i for i in range(g + 1))
+            td = int(np.sum(mask_c[0::2])) * ta + int(np.sum(mask_c[1::2])) * tm
+            return 1e3 * e / (g * td + sh.n_layers * (ta + tm))
+        ranked = sorted(((max(predicted(dcands[i], float(dalphas[i]), g) for g in range(1, tpt_d + 1)),
+                          max(range(1, tpt_d + 1), key=lambda g: predicted(dcands[i], float(dalphas[i]), g)), i)
+                         for i in range(len(djs))), reverse=True)
+        checks = []
+        for pred, g, i in ranked[:3]:
+            mc = np.ascontiguousarray(dcands[i], np.uint8)
+            p = ks.KsSpecParams(int(g), 0, mc.ctypes.data_as(ks.C.POINTER(ks.C.c_uint8)), lat, 0.0, 1, 0)
+            (o, sst, _a), t = timed(lambda: ks.ks_generate_speculative(h, p, e2e_tokens))
+            n_tok = int(sst.steps + sst.accepted)
+            checks.append({"skipped_weight": int(djs[i]), "gamma": int(g), "alpha_hat": float(dalphas[i]),
+                           "alpha": float(sst.accepted) / max(1, sst.drafted),
+                           "predicted_tokens_per_s": pred, "tokens_per_s": n_tok / t})
+        sweep.append({"policy": "Eq. 3 prediction vs measurement for the DP's three best candidates",
+                      "candidates": checks, "greedy_predicted_tokens_per_s": 1e3 / (sh.n_layers * (ta + tm))})
         # sampling mode (Sec. 2.1; nucleus sampling with T 0.7, top-k 50, top-p 0.95 as in Sec. 4)
         p = ks.KsSpecParams(gamma, 1, None, lat, float(args.budget_frac), int(args.resolve_every), 0, 0, 0, 0.0,
                             ks.sampling(0.7, 50, 0.95, 12345))
@@ -484,7 +551,9 @@ def gpu_arm(args):
             "ar_tokens_per_s_device": ar_dev,
             "spec_vs_ar_device": (tok_all / (ms_max * 1e-3)) / ar_dev,
             "lossless_vs_ar": lossless,
-            "latency_model_ms": {"c1": c1, "c2": c2, "c3": c3},
+            "latency_model_ms": {"c1": c1, "c2": c2, "c3": c3,
+                                 "fit": "App. C least squares over attention at n = " + ",".join(map(str, sweep_n)),
+                                 "attention_ms_at_n": [round(t, 5) for t in sweep_t], "fixed_attn_kernels_ms": fixed},
             "prefill_s": t_prefill, "setup_s": t_setup,
             "e2e": {"value": e2e_tok / e2e_s, "unit": UNIT,
                     "h2d_bytes_per_step": (h2d1 - h2d0) / max(1, est.steps),

@@ -116,6 +116,18 @@ typedef struct {
     const int32_t* units;
 } ks_latency;
 
+/* Least-squares fit of the App. C latency model from a profiling sweep:
+ * (c2, c3) minimise sum_k (c2 n[k] + c3 - t_attn[k])^2 over count >= 2
+ * samples (n: context lengths, not all equal; t_attn: the Attn sublayer's
+ * time at n[k]); c1 = mean of t_mlp[0 .. count_mlp - 1] (the MLP sublayer's
+ * time, which does not depend on n).  The coefficients of the model are
+ * non-negative: a negative intercept is refitted through the origin (c3 = 0),
+ * a negative slope gives c2 = 0 and c3 = mean(t_attn).  Writes a kind-0 model
+ * into *out.  Host arrays; no GPU work.  KS_ERR_INVALID_ARG on too few or
+ * non-finite samples, equal context lengths, or a non-positive c1. */
+ks_status ks_fit_latency(const double* n, const double* t_attn, int32_t count, const double* t_mlp,
+                         int32_t count_mlp, ks_latency* out);
+
 typedef struct ks_model ks_model;
 
 /* ------------------------------------------------------------ model (a1-a3) */
@@ -410,7 +422,7 @@ ks_status ks_debug_read(ks_model* m, int32_t what, int32_t layer, int32_t start,
 /* Per-kernel timing with CUDA events on the model's stream.  While enabled,
  * every launch of the kernel class `klass` (0 QKV, 1 attention, 2 merge,
  * 3 O-proj, 4 gate/up, 5 down, 6 LM head, 7 embed, 8 accept, 9 chained
- * projections) is bracketed by events; ks_kernel_time returns the launches
+ * projections, 10 bf16 attention query prep) is bracketed by events; ks_kernel_time returns the launches
  * and total milliseconds since enabling.  Enabling resets the counters.
  * bf16 models run the projections between two attention cores as one chained
  * launch (class 9); while any of classes 0, 3, 4, 5, 6 is enabled they run

@@ -108,6 +108,13 @@ int sm_count();
 
 // ------------------------------------------------------------- attention
 struct AttnArgs {
+    // bf16: TMA map of the whole KV cache viewed as rows of hd elements
+    // ([L][K, V][hk][max_seq] rows; 16-row boxes of hd / 64 swizzled 64-column
+    // chunks, make_weight_map), and the first row of this layer's K and V
+    CUtensorMap kvmap;
+    int kv_row_k, kv_row_v;
+    __nv_bfloat16* q;       // bf16: prepared queries [hk][G R][hd] (QK-norm, RoPE, log2(e)/sqrt(hd))
+    int* err;               // device status word (bf16 kernels: a bounded wait gave up)
     const float* qkv;       // [R][(hq + 2 hk) hd] fp32 projections (pre-norm, pre-RoPE)
     int qkv_ld;
     int R;
@@ -127,6 +134,9 @@ struct AttnArgs {
     const int* stop;        // draft passes: skipped when *stop != 0 (null: always run)
 };
 
+// bf16: queries of the pass prepared once (q) and the new rows' K/V written
+// to the cache; the attention kernel then only streams the cache.
+cudaError_t launch_attn_prep(const AttnArgs& a, cudaStream_t s);
 cudaError_t launch_attention(int dtype, const AttnArgs& a, cudaStream_t s);
 cudaError_t launch_attn_merge(int dtype, const AttnArgs& a, cudaStream_t s);
 // Fixed partition of the key axis for split-KV attention (absolute positions):

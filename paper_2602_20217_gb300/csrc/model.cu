@@ -32,8 +32,8 @@ void set_error(const char* fmt, ...) {
 
 
 constexpr int kSelectCap = 65535;
-constexpr int kKlasses = 10;
-enum { K_QKV = 0, K_ATTN, K_MERGE, K_OPROJ, K_GATEUP, K_DOWN, K_LMHEAD, K_EMBED, K_ACCEPT, K_CHAIN };
+constexpr int kKlasses = 11;
+enum { K_QKV = 0, K_ATTN, K_MERGE, K_OPROJ, K_GATEUP, K_DOWN, K_LMHEAD, K_EMBED, K_ACCEPT, K_CHAIN, K_PREP };
 
 // ------------------------------------------------------------ small kernels
 // x[r] = embed[tok[r]] (fp32); optionally copied to the history plane 0.
@@ -181,7 +181,7 @@ static size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 struct Layout {
     size_t kv, rope, x, ss, xg, qkv, attn_out, act, attn_part, gemv_part, counters, logits, amax_val,
         amax_idx, tok, hist, hist_snap, hist_idx, sims, mask, obj, wts, select, chain_ctr, best, tpt_masks,
-        tpt_tok, tpt_info, tpt_out, dyn, samp, slice, total;
+        tpt_tok, tpt_info, tpt_out, dyn, samp, slice, qbuf, total;
     int n_chunks_max;
     size_t gemv_part_floats;
     int counters_n;
@@ -201,6 +201,9 @@ static bool config_ok(const ks_config* c) {
     if (c->d_model > 64 * 512 || c->d_ff > 64 * 1024) return false;
     if (c->vocab < 1) return false;
     if (c->dtype != KS_DTYPE_F32 && c->dtype != KS_DTYPE_BF16) return false;
+    // bf16 attention addresses cache rows with 32-bit TMA coordinates
+    if (c->dtype == KS_DTYPE_BF16 && 2.0 * c->n_layers * c->n_kv_heads * (double)c->max_seq > 2147483647.0)
+        return false;
     if (c->max_seq < 2 || c->max_rows < 2 || c->max_rows > 16) return false;
     if (c->hist_steps < 1 || c->hist_steps > 64) return false;
     if (c->hist_init_rows < 1 || c->hist_init_rows > c->max_rows) return false;
@@ -274,6 +277,8 @@ static Layout make_layout(const ks_config* c) {
     L.samp = take(2 * ((size_t)R * kSampleMaxK * (sizeof(int) + sizeof(float)) + sizeof(int) * R));
     // chain kernel K-slices: partial sums [2][640][2][16][16] floats, then tickets [2][640]
     L.slice = take(sizeof(float) * 2 * kChainSliceMaxItems * 512 + sizeof(int) * 2 * kChainSliceMaxItems);
+    // bf16 attention: the pass's prepared queries [hk][G R][hd]
+    L.qbuf = take(sizeof(__nv_bfloat16) * (size_t)R * c->n_q_heads * hd);
     L.total = off;
     return L;
 }
@@ -323,6 +328,8 @@ struct ks_model {
     int* n_drafted;           // dynamic exit: draft passes of the step that ran
     float* slice_part;        // chain kernel: K-slice partial sums
     int* slice_ticket;
+    __nv_bfloat16* qbuf;      // bf16 attention: prepared queries of the pass
+    CUtensorMap map_kv;       // bf16 attention: the KV cache as rows of hd elements
     bool last_dynamic = false;
     bool last_sampled = false;   // the drafts on the device were sampled (ks_draft_sample)
     int *q_ids, *q_n, *p_ids, *p_n;   // sampling mode: draft / target distributions [16][kSampleMaxK]
@@ -505,6 +512,14 @@ static ks_status forward(ks_model* m, const int32_t* tok, int R, int p0, const u
         at.part = m->attn_part; at.n_chunks_max = m->lay.n_chunks_max;
         at.out = m->attn_out; at.out_ld = c.n_q_heads * hd;
         at.stop = stop;
+        at.err = m->err;
+        if (bf) {
+            at.kvmap = m->map_kv;
+            at.kv_row_k = 2 * l * c.n_kv_heads * c.max_seq;
+            at.kv_row_v = (2 * l + 1) * c.n_kv_heads * c.max_seq;
+            at.q = m->qbuf;
+            KS_TRY(launch(m, K_PREP, [&] { return launch_attn_prep(at, s); }, "attention query prep"));
+        }
         KS_TRY(launch(m, K_ATTN, [&] { return launch_attention(dt, at, s); }, "attention"));
         KS_TRY(launch(m, K_MERGE, [&] { return launch_attn_merge(dt, at, s); }, "attention merge"));
         return KS_OK;
@@ -786,6 +801,7 @@ ks_status ks_model_create(const ks_config* cfg, const ks_weights* w, void* works
     m->n_drafted = m->rows + (3 * cfg->max_rows + 6);
     m->slice_part = reinterpret_cast<float*>(b + lay.slice);
     m->slice_ticket = reinterpret_cast<int*>(m->slice_part + (size_t)2 * kChainSliceMaxItems * 512);
+    m->qbuf = reinterpret_cast<__nv_bfloat16*>(b + lay.qbuf);
     {
         char* sb = b + lay.samp;
         const size_t RK = (size_t)cfg->max_rows * kSampleMaxK;
@@ -816,6 +832,10 @@ ks_status ks_model_create(const ks_config* cfg, const ks_weights* w, void* works
             ok = ok && make_weight_map(&m->map_down[l], m->w_down[l], d, F, 16);
         }
         ok = ok && make_weight_map(&m->map_lm, m->lm_head, cfg->vocab, d, 16);
+        // [L][K, V][hk][max_seq] rows of hd elements; a box is one 16-key tile
+        ok = ok && make_weight_map(&m->map_kv, m->kv,
+                                   2 * (uint64_t)L * cfg->n_kv_heads * (uint64_t)cfg->max_seq, cfg->head_dim,
+                                   cfg->head_dim / 64);
         for (int b = 0; b < R; ++b) {
             ok = ok && make_stage_map(&m->map_xg[b], m->xg, R, d, b + 1, 4);
             ok = ok && make_stage_map(&m->map_xg2[b], m->xg, R, d, b + 1, 2);
@@ -862,6 +882,11 @@ ks_status ks_model_create(const ks_config* cfg, const ks_weights* w, void* works
     }
     e = cudaMemsetAsync(m->counters, 0, sizeof(int) * lay.counters_n, m->stream);
     if (e != cudaSuccess) return fail(e, "counter reset");
+    // The bf16 attention streams whole 16-key tiles; keys past a row's
+    // position are masked (softmax weight exactly 0), which needs finite
+    // values there: positions never written hold zeros.
+    e = cudaMemsetAsync(m->kv, 0, lay.rope - lay.kv, m->stream);
+    if (e != cudaSuccess) return fail(e, "KV cache reset");
     e = cudaMemsetAsync(m->chain_ctr, 0, sizeof(int) * 2 * chain_counter_ints(), m->stream);
     if (e != cudaSuccess) return fail(e, "counter reset");
     e = cudaMemsetAsync(m->best, 0, sizeof(unsigned long long) * 16, m->stream);

@@ -434,6 +434,62 @@ extern "C" ks_status ks_cosine(const void* X, const void* Y, int32_t dtype, int6
     return KS_OK;
 }
 
+extern "C" ks_status ks_fit_latency(const double* n, const double* t_attn, int32_t count, const double* t_mlp,
+                                    int32_t count_mlp, ks_latency* out) {
+    if (!n || !t_attn || !t_mlp || !out || count < 2 || count_mlp < 1) {
+        set_error("ks_fit_latency: need at least two attention points and one MLP time");
+        return KS_ERR_INVALID_ARG;
+    }
+    // App. C: t_Attn(n) = c2 n + c3 by least squares, t_MLP = c1 (the mean)
+    double sn = 0.0, st = 0.0, c1 = 0.0;
+    for (int k = 0; k < count; ++k) {
+        if (!std::isfinite(n[k]) || !std::isfinite(t_attn[k]) || n[k] < 0.0) {
+            set_error("ks_fit_latency: bad sample %d", k);
+            return KS_ERR_INVALID_ARG;
+        }
+        sn += n[k];
+        st += t_attn[k];
+    }
+    for (int k = 0; k < count_mlp; ++k) c1 += t_mlp[k];
+    c1 /= count_mlp;
+    const double nb = sn / count, tb = st / count;
+    double sxx = 0.0, sxy = 0.0;
+    for (int k = 0; k < count; ++k) {
+        sxx += (n[k] - nb) * (n[k] - nb);
+        sxy += (n[k] - nb) * (t_attn[k] - tb);
+    }
+    if (!(sxx > 0.0)) {
+        set_error("ks_fit_latency: the context lengths must not all be equal");
+        return KS_ERR_INVALID_ARG;
+    }
+    double c2 = sxy / sxx, c3 = tb - c2 * nb;
+    // the model's coefficients are non-negative: a negative intercept refits
+    // through the origin, a negative slope leaves the mean as the intercept
+    if (c3 < 0.0) {
+        double snn = 0.0, snt = 0.0;
+        for (int k = 0; k < count; ++k) {
+            snn += n[k] * n[k];
+            snt += n[k] * t_attn[k];
+        }
+        c2 = snt / snn;
+        c3 = 0.0;
+    }
+    if (c2 < 0.0) {
+        c2 = 0.0;
+        c3 = tb;
+    }
+    if (!(c1 > 0.0) || !std::isfinite(c1) || !std::isfinite(c2) || !std::isfinite(c3)) {
+        set_error("ks_fit_latency: the fitted model is not valid (t_MLP must be positive)");
+        return KS_ERR_INVALID_ARG;
+    }
+    out->kind = 0;
+    out->c1 = c1;
+    out->c2 = c2;
+    out->c3 = c3;
+    out->units = nullptr;
+    return KS_OK;
+}
+
 extern "C" size_t ks_select_scratch_bytes(int32_t n_sublayers, int32_t budget_units) {
     if (n_sublayers < 2 || n_sublayers > kMaxItems || budget_units < 0 || budget_units > 65535) return 0;
     return select_scratch_bytes(n_sublayers, budget_units);

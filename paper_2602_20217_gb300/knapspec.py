@@ -19,7 +19,7 @@ KS_OK, KS_ERR_INVALID_ARG, KS_ERR_CUDA, KS_ERR_WORKSPACE, KS_ERR_CAPACITY, KS_ER
     KS_ERR_UNSUPPORTED, KS_ERR_STATE = range(8)
 KS_DTYPE_F32, KS_DTYPE_BF16 = 0, 1
 KLASS = {"qkv": 0, "attn": 1, "merge": 2, "oproj": 3, "gateup": 4, "down": 5, "lmhead": 6,
-         "embed": 7, "accept": 8, "chain": 9}
+         "embed": 7, "accept": 8, "chain": 9, "prep": 10}
 
 
 class KsConfig(C.Structure):
@@ -96,6 +96,8 @@ _SIGS = {
                             C.c_void_p, C.c_void_p, C.c_void_p]),
     "ks_history_similarities": (C.c_int, [C.c_void_p, C.c_void_p, C.POINTER(C.c_int32)]),
     "ks_select_scratch_bytes": (C.c_size_t, [C.c_int32, C.c_int32]),
+    "ks_fit_latency": (C.c_int, [C.POINTER(C.c_double), C.POINTER(C.c_double), C.c_int32, C.POINTER(C.c_double),
+                                 C.c_int32, C.POINTER(KsLatency)]),
     "ks_select_mask": (C.c_int, [C.POINTER(KsLatency), C.c_void_p, C.c_int64, C.c_int32, C.c_int32, C.c_void_p,
                                  C.c_void_p, C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p]),
     "ks_select_mask_static": (C.c_int, [C.POINTER(KsLatency), C.c_void_p, C.c_int64, C.c_int32, C.c_int32,
@@ -332,6 +334,18 @@ def latency(kind: int = 0, c1: float = 0.0, c2: float = 0.0, c3: float = 0.0, un
         u = np.ascontiguousarray(units, dtype=np.int32)
     lat = KsLatency(kind, c1, c2, c3, u.ctypes.data_as(C.POINTER(C.c_int32)) if u is not None else None)
     return lat, u
+
+
+def ks_fit_latency(ns, t_attn, t_mlp):
+    """App. C least-squares fit in the library: returns a kind-0 KsLatency."""
+    n = np.ascontiguousarray(ns, np.float64)
+    ta = np.ascontiguousarray(t_attn, np.float64)
+    tm = np.ascontiguousarray(np.atleast_1d(t_mlp), np.float64)
+    out = KsLatency()
+    check(load().ks_fit_latency(n.ctypes.data_as(C.POINTER(C.c_double)), ta.ctypes.data_as(C.POINTER(C.c_double)),
+                                len(n), tm.ctypes.data_as(C.POINTER(C.c_double)), len(tm), C.byref(out)),
+          "ks_fit_latency")
+    return out
 
 
 def ks_select_scratch_bytes(n_sublayers: int, budget_units: int) -> int:

@@ -168,3 +168,32 @@ def test_product_path_fails_loudly_without_library(tmp_path):
             ks.load(str(tmp_path / "missing.so"))
     finally:
         ks._lib = saved
+
+
+def test_fit_latency_matches_the_oracle_fit(lib):
+    """App. C's least-squares fit in the library equals the oracle's
+    (np.linalg.lstsq) fit, and the non-negativity rules apply."""
+    from oracle import select as S
+    from paper_2602_20217_gb300 import knapspec as ks
+    rng = np.random.default_rng(4)
+    ns = np.array([4096, 8192, 16384, 32768, 65536], np.float64)
+    t_attn = 0.01 + 6.9e-7 * ns + rng.normal(0, 1e-4, len(ns))
+    t_mlp = 0.16 + rng.normal(0, 1e-3, 3)
+    got = ks.ks_fit_latency(ns, t_attn, t_mlp)
+    c1, c2, c3 = S.fit_latency(ns, t_attn, t_mlp)
+    assert got.kind == 0
+    assert got.c1 == pytest.approx(c1, rel=1e-12)
+    assert got.c2 == pytest.approx(c2, rel=1e-9)
+    assert got.c3 == pytest.approx(c3, rel=1e-9)
+    # a negative intercept: refitted through the origin
+    got = ks.ks_fit_latency([1000.0, 2000.0, 3000.0], [0.9, 2.0, 3.1], [0.5])
+    assert got.c3 == 0.0
+    assert got.c2 == pytest.approx((1000 * 0.9 + 2000 * 2.0 + 3000 * 3.1) / (1000 ** 2 + 2000 ** 2 + 3000 ** 2))
+    # a negative slope: the mean time as the intercept
+    got = ks.ks_fit_latency([1000.0, 2000.0], [0.3, 0.2], [0.5])
+    assert got.c2 == 0.0 and got.c3 == pytest.approx(0.25)
+    # too few points, equal lengths, non-positive MLP time
+    for args in [([1.0], [1.0], [1.0]), ([5.0, 5.0], [1.0, 2.0], [1.0]), ([1.0, 2.0], [1.0, 2.0], [0.0])]:
+        with pytest.raises(ks.KsError):
+            ks.ks_fit_latency(*args)
+
