@@ -603,8 +603,8 @@ def main():
     ap.add_argument("--tpt-candidates", dest="tpt_candidates", type=int, default=8)
     ap.add_argument("--tau-conf", dest="tau_conf", type=float, default=0.0,
                     help="dynamic drafting exit threshold (Sec. 3.5); 0 drafts gamma tokens every step")
-    ap.add_argument("--tpt-max-gamma", dest="tpt_max_gamma", type=int, default=7,
-                    help="D of Alg. 2 (1..15); the default keeps verify passes at 8 rows or fewer")
+    ap.add_argument("--tpt-max-gamma", dest="tpt_max_gamma", type=int, default=10,
+                    help="D of Alg. 2 (1..15; the paper's is 10)")
     ap.add_argument("--clocks-dir", dest="clocks_dir", default="",
                     help="directory for the raw clock samples of the timed region (default: the temp dir)")
     ap.add_argument("--sweep", action="store_true",

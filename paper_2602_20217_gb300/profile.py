@@ -44,7 +44,7 @@ def main():
     m = Model(sh, max_seq=args.prompt + (args.steps + 2) * (args.gamma + 1) + 16, seed=wl.weight_seed)
     m.prefill(prompt)
     if args.timing:
-        for k in range(10):   # every class: the projections then run one per launch
+        for k in ks.KLASS.values():   # every class: the projections then run one per launch
             ks.ks_kernel_timing(m.h, k, True)
     mask = np.array([0, 1] * sh.n_layers, np.uint8)   # draft: MLP sublayers only
     torch.cuda.synchronize()
