@@ -487,10 +487,14 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
         // ------------------------------------------------------ consumers
         float acc[kChains][NT][4], accu[kChains][NT][4];
         bool failed = false;
+        // A wait of one consumer warp that gives up is acted on by all four
+        // together at the next stage's barrier (they must leave the loop
+        // together: a warp left behind at the named barrier would wait forever).
+        bool gave_up = false;
         int n_items = 0;   // items finished by this CTA (selects the partials buffer)
         for (int t = 0;; ++t) {
             const int slot = t % S;
-            const bool ok = mbar_wait(&full[slot], (uint32_t)((t / S) & 1), kWaitLimitNs);
+            const bool ok = !gave_up && mbar_wait(&full[slot], (uint32_t)((t / S) & 1), kWaitLimitNs);
             if (consumers_or(!ok)) {
                 failed = true;
                 break;
@@ -548,8 +552,8 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
                         accu[0][nt][i] += accu[c][nt][i];
                     }
             if (n_items >= 2 && !mbar_wait(&red_free[b], (uint32_t)(((n_items >> 1) - 1) & 1), kWaitLimitNs)) {
-                failed = true;
-                break;
+                gave_up = true;   // leave at the next barrier, with the other warps
+                continue;
             }
 #pragma unroll
             for (int nt = 0; nt < NT; ++nt)
