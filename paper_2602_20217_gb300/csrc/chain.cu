@@ -367,7 +367,7 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
             int k = 0;
             Phase P = decode(a, 0);
             int it = (int)blockIdx.x;
-            while (ok) {   // `it` counts units: item it / n_sl, K-slice it % n_sl
+            while (ok) {   // `it` counts units: K-slice it / n_items, item it % n_items
                 if (it >= P.n_units) {
                     if (++k >= a.n_phases) break;
                     P = decode(a, k);
@@ -378,7 +378,10 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
                 // ticket is first needed at the unit's last stage, so its
                 // round trip overlaps the unit's other stages)
                 const int next = P.n_units > grid ? grid + atomicAdd(&queue[k], 1) : INT_MAX;
-                const int item = it / P.n_sl, sl = it - item * P.n_sl;
+                // slice-major: every item's first K-slice comes before any
+                // second one, so the units taken first (one per CTA) read the
+                // previous phase's first blocks, which complete first
+                const int sl = it / P.n_items, item = it - sl * P.n_items;
                 const int kt0 = sl * P.sl_len, kt1 = min(P.tpi, kt0 + P.sl_len);
                 for (int kt = kt0; kt < kt1 && ok; ++kt)
                     ok = issue(k, P, item, kt, sl, kt == kt1 - 1 && next >= P.n_units);
