@@ -137,9 +137,14 @@ typedef struct ks_model ks_model;
 size_t ks_workspace_bytes(const ks_config* cfg);
 
 /* Validate cfg, borrow the weights and the workspace (dev, 256-byte aligned,
- * at least ks_workspace_bytes(cfg) bytes), build the RoPE table, and return a
- * handle bound to `stream` (a cudaStream_t; NULL = legacy default stream).
- * No decoding state exists until ks_prefill. */
+ * at least ks_workspace_bytes(cfg) bytes), build the RoPE table, zero the KV
+ * cache region of the workspace (the attention streams whole 16-key tiles,
+ * and keys past a row's position get an exact zero weight only if their
+ * values are finite), and return a handle bound to `stream` (a cudaStream_t;
+ * NULL = legacy default stream); the call waits for the stream.  bf16
+ * configs need 2 n_layers n_kv_heads max_seq < 2^31 (32-bit cache-row
+ * coordinates); ks_workspace_bytes returns 0 otherwise.  No decoding state
+ * exists until ks_prefill. */
 ks_status ks_model_create(const ks_config* cfg, const ks_weights* w, void* workspace,
                           size_t workspace_bytes, void* stream, ks_model** out);
 ks_status ks_model_destroy(ks_model* m);
