@@ -291,9 +291,11 @@ KS_DEV float fast_exp2(float x) {
 }
 
 
+// One CTA's work: query rows q0 .. q0 + 8 NQ - 1 of KV head h over one chunk.
+// `a` is the kernel's parameter (its tensor map is read in place by TMA).
 template <int HD, int NQ>
-__global__ void __launch_bounds__(128, kAttnCtasPerSm) attn_bf16_kernel(const __grid_constant__ AttnArgs a) {
-    if (a.stop && *a.stop) return;   // a draft pass after the dynamic exit
+__device__ __forceinline__ void attn_bf16_body(const AttnArgs& a, int h, int q0, unsigned char* smem_raw,
+                                               uint64_t (*full)[kWarpStages]) {
     constexpr int P = HD + 8;          // Qs row pitch (bf16)
     constexpr int KD = HD / 16;        // k-steps of K Q^T = dim tiles of V^T P^T
     constexpr int QR = 8 * NQ;         // query rows per round
@@ -302,17 +304,13 @@ __global__ void __launch_bounds__(128, kAttnCtasPerSm) attn_bf16_kernel(const __
     constexpr int RING = kWarpStages * STAGE;        // one warp's ring
     constexpr int OP = HD + 4;         // pitch of a query row in the combine area (fp32)
     static_assert(QR * (OP + 2) * 4 <= RING, "combine area exceeds the warp's ring");
-    extern __shared__ unsigned char smem_raw[];
     // 1024-byte aligned: the swizzle pattern repeats every 1024 bytes
     unsigned char* rings = reinterpret_cast<unsigned char*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
     __nv_bfloat16* Qs = reinterpret_cast<__nv_bfloat16*>(rings + kAttnWarps * RING);   // [QR][P]
-    __shared__ __align__(8) uint64_t full[kAttnWarps][kWarpStages];
 
     const int G = a.hq / a.hk;
     const int M = G * a.R;
-    const int rounds = (M + QR - 1) / QR;
-    const int h = (int)blockIdx.x / rounds, rd = (int)blockIdx.x - h * rounds;
     const int c = my_chunk(a);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int g = lane >> 2, t = lane & 3;
@@ -351,7 +349,6 @@ __global__ void __launch_bounds__(128, kAttnCtasPerSm) attn_bf16_kernel(const __
         while (issued < pre) issue(issued++);
 
     // queries of this round, rows m = q0 + row (rows past M are zero)
-    const int q0 = rd * QR;
     constexpr int CPR = HD / 8;      // 16-byte pieces per row
     for (int j = tid; j < QR * CPR; j += blockDim.x) {
         const int row = j / CPR, col = (j - row * CPR) * 8;
@@ -580,6 +577,28 @@ __global__ void __launch_bounds__(128, kAttnCtasPerSm) attn_bf16_kernel(const __
         *reinterpret_cast<float4*>(a.part + (((size_t)r * a.hq + h * G + gq) * a.n_chunks_max + c) * (HD + kPartPad) +
                                    kPartPad + d4) = O;
     }
+}
+
+// Query rows m = r G + gq in rounds of 8 NQ rows, one round per CTA (the
+// rounds of a KV head adjacent in x).  A last round with at most 8 (NQ - 1)
+// rows (the second round of 40 rows at eight query heads per KV head) runs
+// with one query tile less; a row's arithmetic is the same in either.
+template <int HD, int NQ>
+__global__ void __launch_bounds__(128, kAttnCtasPerSm) attn_bf16_kernel(const __grid_constant__ AttnArgs a) {
+    if (a.stop && *a.stop) return;   // a draft pass after the dynamic exit
+    extern __shared__ unsigned char smem_raw[];
+    __shared__ __align__(8) uint64_t full[kAttnWarps][kWarpStages];
+    constexpr int QR = 8 * NQ;
+    const int M = (a.hq / a.hk) * a.R;
+    const int rounds = (M + QR - 1) / QR;
+    const int h = (int)blockIdx.x / rounds, q0 = ((int)blockIdx.x - h * rounds) * QR;
+    if constexpr (NQ > 1) {
+        if (M - q0 <= 8 * (NQ - 1)) {
+            attn_bf16_body<HD, NQ - 1>(a, h, q0, smem_raw, full);
+            return;
+        }
+    }
+    attn_bf16_body<HD, NQ>(a, h, q0, smem_raw, full);
 }
 
 // ----------------------------------------------------------- fp32 kernel
