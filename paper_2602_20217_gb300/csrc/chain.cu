@@ -16,16 +16,16 @@
 //  * warp 4 (weights): claims work items phase by phase from per-phase
 //    atomic queues (16 output features over the full K) and issues their
 //    2-D TMA weight boxes into a ring of shared-memory stages;
-//  * warp 5 (activations): follows the same stage sequence; on entering a
-//    phase it waits until the previous phase's done-counter reaches its item
-//    count, computes the per-row 1/rms of the residual (normalised inputs),
-//    and then issues the activation boxes of each stage;
+//  * warp 5 (activations): follows the same stage sequence; before a stage
+//    it waits until the block of the previous phase's output that the stage
+//    reads is complete, then issues the stage's activation boxes;
 //  * warps 0-3 (consumers): mma.sync m16n8k16 with weights as A and the R
 //    activation rows as B (columns independent: batch invariant), each warp
 //    a quarter of every stage's columns,
 //    then hand each item's per-warp sums to
-//  * warp 6 (epilogue): adds them in warp order (fixed), runs the fused
-//    epilogue, and after the CTA's last item of a phase adds its item count
+//  * warp 6 (epilogue): adds them in warp order (fixed), computes the rows'
+//    1/rms at its first item of a normed phase (normalised inputs), runs the
+//    fused epilogue, and after the CTA's last item of a phase adds its item count
 //    to the phase's done-counter (one release per CTA and phase).  LM head:
 //    each CTA keeps its best (logit, id) per row and merges it into a 64-bit
 //    key with atomicMax (value first, then the lower id: any merge order gives
@@ -264,6 +264,42 @@ KS_DEV void epilogue(const ChainArgs& a, const Phase& P, int k, int it, float (&
     }
 }
 
+// 1 / rms of each of the R rows from the 16-feature partial sums of squares
+// of the residual (ss[group][row]): lane l adds groups l, l + 32, ... in that
+// order, then a butterfly, and lane 0's total is used; the same order for
+// every R.  A group's row sums are contiguous, so all rows load together.
+template <int NT>
+KS_DEV void row_scales(const ChainArgs& a, int lane, float* out) {
+    constexpr int kRows = NT * 8;
+    const int R = a.R;   // <= kRows
+    const int groups = (a.d + 15) >> 4;
+    float s[kRows];
+#pragma unroll
+    for (int r = 0; r < kRows; ++r) s[r] = 0.f;
+#pragma unroll 2
+    for (int q = lane; q < groups; q += 32) {
+        const float4* src = reinterpret_cast<const float4*>(a.ss + (size_t)q * kMaxRows);
+#pragma unroll
+        for (int v = 0; v < kRows / 4; ++v) {
+            if (4 * v < R) {
+                const float4 f = __ldcg(src + v);
+                s[4 * v] += f.x;
+                s[4 * v + 1] += f.y;
+                s[4 * v + 2] += f.z;
+                s[4 * v + 3] += f.w;
+            }
+        }
+    }
+#pragma unroll
+    for (int r = 0; r < kRows; ++r) {
+        if (r < R) {
+            const float t = warp_sum(s[r]);
+            if (lane == 0) out[r] = rsqrtf(t / (float)a.d + a.eps);
+        }
+    }
+    __syncwarp();
+}
+
 template <int NT, int CTAS_PER_SM>
 __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __grid_constant__ ChainArgs a) {
     // A draft pass after the dynamic exit: nothing to do.  The flag only
@@ -280,7 +316,7 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
     __shared__ int slot_last[kMaxStages];   // the stage ends this CTA's last item of its phase
     __shared__ int slot_sl[kMaxStages];     // the item's K-slice
     __shared__ float ones[kMaxRows];        // the input scale of phases without a norm
-    __shared__ float scale[2][kMaxRows];
+    __shared__ float scale[kMaxRows];       // 1 / rms of the rows (epilogue warp only)
     __shared__ float red[2][4][2][NT * 4][32];   // [buffer][consumer warp][gate, up][fragment][lane]
     __shared__ int red_k[2], red_it[2], red_last[2], red_sl[2];
     __shared__ __align__(8) uint64_t red_full[2];   // 4 consumer warps arrive
@@ -407,7 +443,7 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
         // ---------------------------------------------- activation loader
         grid_dependency_wait();   // the first phase's input comes from the previous kernel
         int cur = -1, ready = 0;
-        bool scaled = false, ok = true;
+        bool ok = true;
         for (int t = 0;; ++t) {
             const int slot = t % S;
             // lane 0 waits; the shuffle broadcasts the outcome and orders the
@@ -438,7 +474,6 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
             if (k != cur) {
                 cur = k;
                 ready = 0;      // blocks of phase k - 1 known to be complete
-                scaled = false;
             }
             if (k > 0 && kt >= ready) {
                 // wait for the block of phase k - 1 that this stage reads
@@ -453,26 +488,6 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
                 }
                 fence_proxy_async_global();
                 if (kt == ready) ++ready;   // stages of an item come in order
-            }
-            // The 1/rms scale needs all of phase k - 1: ready when this item's
-            // last stage had its block (an item's stages cover every block).
-            if (!scaled && kt == P.tpi - 1) {
-                scaled = true;
-                if (normed_input(P.kind)) {
-                    // 1 / rms of each row from the 16-feature partial sums of
-                    // squares: lane l adds groups l, l + 32, ..., then a
-                    // butterfly; the same order for every R
-                    const int groups = (a.d + 15) >> 4;
-                    for (int r = 0; r < R; ++r) {
-                        float s = 0.f;
-                        for (int q = lane; q < groups; q += 32) s += __ldcg(&a.ss[q * kMaxRows + r]);
-                        s = warp_sum(s);
-                        if (lane == 0) scale[k & 1][r] = rsqrtf(s / (float)a.d + a.eps);
-                    }
-                } else if (lane < kMaxRows) {
-                    scale[k & 1][lane] = 1.f;
-                }
-                __syncwarp();
             }
             if (lane == 0) {
                 const int nb = (P.kind == CH_GU) ? 2 : 4;
@@ -590,6 +605,7 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
                 run_i[nt][c] = INT_MAX;
             }
         int items_in_phase = 0;   // items of the current phase finished by this CTA
+        int scale_k = -1;         // the phase whose row scales `scale` holds
         bool ok = true;
         for (int n = 0;; ++n) {
             const int b = n & 1;
@@ -660,8 +676,16 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
                         }
                 }
             }
+            if (complete && normed_input(P.kind) && k != scale_k) {
+                // This CTA's first item of a normed phase: its last stage
+                // waited for every block of phase k - 1 (an item's stages
+                // cover them all), so every row group's partial sums of
+                // squares are written.
+                scale_k = k;
+                row_scales<NT>(a, lane, scale);
+            }
             if (complete) {
-                epilogue<NT>(a, P, k, it, acc, accu, normed_input(P.kind) ? scale[k & 1] : ones, run_v, run_i);
+                epilogue<NT>(a, P, k, it, acc, accu, normed_input(P.kind) ? scale : ones, run_v, run_i);
                 ++items_in_phase;
             }
             if (complete && k + 1 < a.n_phases) {
