@@ -31,7 +31,10 @@
  *    ks_last_error).  No kernel waits on another launch; the pipeline waits
  *    inside a kernel (TMA barriers) give up after 2 s, record the fact in a
  *    device status word and return, and the next synchronising call reports
- *    KS_ERR_TIMEOUT.
+ *    KS_ERR_TIMEOUT.  The status word stays set until the model is created
+ *    again (every later synchronising call reports it), and the chained
+ *    projection kernels of a job enqueued after it was set return at once, so
+ *    a long job that hit a timeout ends quickly instead of waiting again.
  *  - One handle is used by one host thread at a time and issues all work on
  *    the stream given at creation.
  *  - Greedy argmax ties resolve to the lowest token id.

@@ -300,6 +300,22 @@ KS_DEV void row_scales(const ChainArgs& a, int lane, float* out) {
     __syncwarp();
 }
 
+// One thread per CTA, as the CTA leaves: the last CTA of the launch to leave
+// resets the queues and counters of its counter set for a later launch.
+KS_DEV void count_out(int n_phases, int* queue, int* done, int* exits, int* blocks) {
+    __threadfence();
+    if (atomicAdd(exits, 1) == (int)gridDim.x - 1) {
+        __threadfence();
+        for (int k = 0; k < n_phases; ++k) {
+            queue[k] = 0;
+            done[k] = 0;
+            for (int b = 0; b < kMaxBlocks; ++b) blocks[k * kMaxBlocks + b] = 0;
+        }
+        *exits = 0;
+        __threadfence();
+    }
+}
+
 template <int NT, int CTAS_PER_SM>
 __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __grid_constant__ ChainArgs a) {
     // A draft pass after the dynamic exit: nothing to do.  The flag only
@@ -321,6 +337,7 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
     __shared__ int red_k[2], red_it[2], red_last[2], red_sl[2];
     __shared__ __align__(8) uint64_t red_full[2];   // 4 consumer warps arrive
     __shared__ __align__(8) uint64_t red_free[2];   // the epilogue warp arrives
+    __shared__ int void_job;
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int R = a.R, S = a.stages;
@@ -331,6 +348,13 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
     int* blocks = a.counters + 2 * kChainMaxPhases + 1;   // [phase][kMaxBlocks]
 
     if (tid == 0) {
+        // A job whose status word already holds an error is void (the word
+        // stays set until the model is created again): the CTA skips its
+        // work, so each later launch of the job ends at once instead of
+        // running into bounded waits of its own.  One thread reads the word
+        // (it can change during the launch) and the barrier below hands the
+        // decision to the whole CTA.
+        void_job = __ldcg(a.err) != 0;
         for (int i = 0; i < S; ++i) {
             mbar_init(&full[i], 2);
             mbar_init(&empty[i], 4);
@@ -344,6 +368,10 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
     }
     if (tid < kMaxRows) ones[tid] = 1.f;
     __syncthreads();
+    if (void_job) {   // still counted out, so the launch's counters are reset
+        if (tid == 0) count_out(a.n_phases, queue, done, exits, blocks);
+        return;
+    }
 
     if (warp == kWarpW) {
         // -------------------------------------------------- weight loader
@@ -736,19 +764,7 @@ __global__ void __launch_bounds__(kThreads, CTAS_PER_SM) chain_kernel(const __gr
 
     // the last CTA to leave resets the queues and counters for the next launch
     __syncthreads();
-    if (tid == 0) {
-        __threadfence();
-        if (atomicAdd(exits, 1) == (int)gridDim.x - 1) {
-            __threadfence();
-            for (int k = 0; k < a.n_phases; ++k) {
-                queue[k] = 0;
-                done[k] = 0;
-                for (int b = 0; b < kMaxBlocks; ++b) blocks[k * kMaxBlocks + b] = 0;
-            }
-            *exits = 0;
-            __threadfence();
-        }
-    }
+    if (tid == 0) count_out(a.n_phases, queue, done, exits, blocks);
 }
 
 }  // namespace
