@@ -427,6 +427,15 @@ ks_status ks_generate_speculative(ks_model* m, const ks_spec_params* params, int
 ks_status ks_debug_read(ks_model* m, int32_t what, int32_t layer, int32_t start, int32_t count,
                         void* dst, size_t bytes);
 
+/* Host-side fault injection for tests of the error path: after the model's
+ * stream is idle, write `code` into the device status word, as a kernel
+ * whose bounded wait gave up writes 1 (a self-check failure writes 2..5);
+ * 0 clears the word.  While the word is set, every synchronising call
+ * reports it (1: KS_ERR_TIMEOUT, else KS_ERR_STATE) and the chained
+ * projection kernels of later launches return at once.  Errors: null m,
+ * code outside 0..5 -> KS_ERR_INVALID_ARG; a CUDA failure -> KS_ERR_CUDA. */
+ks_status ks_debug_set_status(ks_model* m, int32_t code);
+
 /* Per-kernel timing with CUDA events on the model's stream.  While enabled,
  * every launch of the kernel class `klass` (0 QKV, 1 attention, 2 merge,
  * 3 O-proj, 4 gate/up, 5 down, 6 LM head, 7 embed, 8 accept, 9 chained

@@ -1851,6 +1851,16 @@ ks_status ks_generate_speculative(ks_model* m, const ks_spec_params* prm, int32_
     return KS_OK;
 }
 
+ks_status ks_debug_set_status(ks_model* m, int32_t code) {
+    if (!m || code < 0 || code > 5) {
+        set_error("ks_debug_set_status: bad argument");
+        return KS_ERR_INVALID_ARG;
+    }
+    KS_CUDA(cudaStreamSynchronize(m->stream), "debug status");
+    KS_CUDA(cudaMemcpy(m->err, &code, sizeof(int32_t), cudaMemcpyHostToDevice), "debug status");
+    return KS_OK;
+}
+
 ks_status ks_debug_read(ks_model* m, int32_t what, int32_t layer, int32_t start, int32_t count, void* dst,
                         size_t bytes) {
     if (!m || !dst) return KS_ERR_INVALID_ARG;

@@ -105,6 +105,7 @@ _SIGS = {
     "ks_generate_speculative": (C.c_int, [C.c_void_p, C.POINTER(KsSpecParams), C.c_int32, C.c_void_p,
                                           C.POINTER(KsSpecStats), C.c_void_p]),
     "ks_debug_read": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32, C.c_int32, C.c_int32, C.c_void_p, C.c_size_t]),
+    "ks_debug_set_status": (C.c_int, [C.c_void_p, C.c_int32]),
     "ks_kernel_timing": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32]),
     "ks_kernel_time": (C.c_int, [C.c_void_p, C.c_int32, C.POINTER(C.c_int64), C.POINTER(C.c_double)]),
     "ks_select_tpt": (C.c_int, [C.c_void_p, C.POINTER(KsLatency), C.c_int32, C.c_int32, C.c_void_p,
@@ -382,6 +383,11 @@ def ks_generate_speculative(h: int, params: KsSpecParams, n_tokens: int):
 def ks_debug_read(h: int, what: int, layer: int, start: int, count: int, out: np.ndarray):
     check(load().ks_debug_read(h, what, layer, start, count, out.ctypes.data, out.nbytes), "ks_debug_read")
     return out
+
+
+def ks_debug_set_status(h: int, code: int):
+    """Host-side fault injection: write `code` into the device status word (0 clears it)."""
+    check(load().ks_debug_set_status(h, int(code)), "ks_debug_set_status")
 
 
 def ks_kernel_timing(h: int, klass: int, enable: bool):
