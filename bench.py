@@ -168,7 +168,7 @@ def reference_arm(args):
             "warmup": args.warmup, "ms_per_step": 1e3 / cb["value"], "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
             "impl": "reference",
-            "config": {"workload": wl, "model": WORKLOADS[wl].shape.name, "prompt": WORKLOADS[wl].prompt_len},
+            "config": {"workload": wl, "prompt": WORKLOADS[wl].prompt_len},
             "cpu_baseline": cb,
             "e2e": {"value": cb["value"], "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -533,7 +533,7 @@ def gpu_arm(args):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_max / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": sh.dtype,
             "data": "synthetic (seeded random-init weights, uniform random prompt ids)",
-            "config": {"workload": wl.name, "model": sh.name, "prompt": wl.prompt_len, "gamma": gamma,
+            "config": {"workload": wl.name, "prompt": wl.prompt_len, "gamma": gamma,
                        "policy": ((f"knapsack re-solved every {args.resolve_every} step(s), "
                                   f"budget {args.budget_frac} of sum w") if args.policy == "knapsack" else
                                  (f"TPT stage every {args.tpt_every} step(s), K {args.tpt_candidates}, "

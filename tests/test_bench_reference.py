@@ -28,6 +28,7 @@ def test_reference_arm_prints_one_contract_line():
     assert d["value"] > 0 and d["higher_is_better"] is True and d["vs_baseline"] is None
     assert d["ms_per_step"] > 0
     assert d["config"]["workload"] == "tiny"
+    assert "model" not in d["config"]   # the workload names the shape
     cb = d["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"] and cb["sample"]
     e = d["e2e"]
